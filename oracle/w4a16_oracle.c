@@ -1,0 +1,196 @@
+/*
+ * CPU oracle for the group-wise int4 weight-only (W4A16) linear layer.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call, link or
+ * load this file: it is used by tests/, by __graft_entry__.smoke() and by
+ * the cpu_baseline / --impl reference legs of bench.py.  It shares no code,
+ * header, table or constant with the CUDA library.
+ *
+ * What it computes.  The paper runs its 175B decoder "4-bit pre-quantized"
+ * with "mixed-precision quantization" (Sec. 3.1, Sec. 4.1) and gives no
+ * format.  The format used here is the one fixed for this library:
+ *   - symmetric int4 per group of g consecutive k, zero point 8,
+ *     stored code q in 0..15;
+ *   - two codes per byte, the even k in bits 0..3, the odd k in bits 4..7;
+ *   - one bf16 scale per (row n, group k/g);
+ *   - dequantised weight wd = RNE_bf16( (q - 8) * s ), one rounding of the
+ *     exact fp32 product;
+ *   - out[m,n] = sum_k x[m,k] * wd[n,k], accumulated here in fp64 with k
+ *     ascending (the reference value that the GPU result is measured against).
+ * The quantiser (data generation): s = RNE_bf16(amax / 7) with an fp32
+ * division, q = clamp(round_half_even(w / s), -8, 7) + 8, all-zero group ->
+ * s = 0 and q = 8.
+ *
+ * Every function is a direct transcription of that definition: no blocking,
+ * no fusion, no reordering.  The bf16 rounding is written out from the IEEE
+ * binary32 bit pattern (round to nearest, ties to even) rather than taken from
+ * any library.
+ */
+#include <stdint.h>
+#include <string.h>
+#include <math.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* ---- bf16 <-> fp32 ----------------------------------------------------- */
+
+/* bf16 is the top 16 bits of an IEEE binary32.  Widening is exact. */
+float oracle_bf16_to_f32(uint16_t h) {
+    uint32_t u = ((uint32_t)h) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+/* Round a binary32 to the nearest bf16, ties to even.  Dropping the low 16
+ * bits is a truncation toward zero of the magnitude; adding 0x7FFF plus the
+ * lowest kept bit before truncating moves every value that lies more than
+ * halfway (or exactly halfway with an odd kept part) up to the next bf16.
+ * A carry out of the mantissa correctly bumps the exponent (and overflows to
+ * infinity).  NaN inputs stay NaN (quiet bit forced, sign kept). */
+uint16_t oracle_bf16_rne(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu) != 0u)
+        return (uint16_t)((u >> 16) | 0x0040u);
+    uint32_t kept_lsb = (u >> 16) & 1u;
+    u += 0x7FFFu + kept_lsb;
+    return (uint16_t)(u >> 16);
+}
+
+/* ---- packing ------------------------------------------------------------ */
+
+/* q[n*K + k] = code of weight (n, k), 0..15. */
+void oracle_unpack(const uint8_t* packed, int64_t N, int64_t K, uint8_t* q) {
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t k = 0; k < K; ++k) {
+            uint8_t b = packed[n * (K / 2) + k / 2];
+            q[n * K + k] = (k % 2 == 0) ? (uint8_t)(b & 0x0F) : (uint8_t)(b >> 4);
+        }
+}
+
+void oracle_pack(const uint8_t* q, int64_t N, int64_t K, uint8_t* packed) {
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t j = 0; j < K / 2; ++j) {
+            uint8_t lo = q[n * K + 2 * j] & 0x0F;
+            uint8_t hi = q[n * K + 2 * j + 1] & 0x0F;
+            packed[n * (K / 2) + j] = (uint8_t)(lo | (hi << 4));
+        }
+}
+
+/* ---- quantiser (input generation) --------------------------------------- */
+
+/* w: fp32 [N, K] row-major.  packed: [N, K/2].  scales: bf16 bits [N, K/g].
+ * Returns 0, or -1 if the shape is not one the format admits. */
+int oracle_quantize(const float* w, int64_t N, int64_t K, int64_t g,
+                    uint8_t* packed, uint16_t* scales) {
+    if (N < 0 || K <= 0 || g <= 0 || K % g != 0 || K % 2 != 0) return -1;
+    int64_t KG = K / g;
+    for (int64_t n = 0; n < N; ++n) {
+        for (int64_t j = 0; j < KG; ++j) {
+            const float* grp = w + n * K + j * g;
+            float amax = 0.0f;
+            for (int64_t t = 0; t < g; ++t) {
+                float a = fabsf(grp[t]);
+                if (a > amax) amax = a;
+            }
+            volatile float seven = 7.0f;           /* keep the division in fp32 */
+            float s_exact = amax / seven;
+            uint16_t s_bits = oracle_bf16_rne(s_exact);
+            float s = oracle_bf16_to_f32(s_bits);
+            scales[n * KG + j] = s_bits;
+            for (int64_t t = 0; t < g; ++t) {
+                int64_t k = j * g + t;
+                int code;
+                if (s == 0.0f) {
+                    code = 8;
+                } else {
+                    float r = nearbyintf(grp[t] / s);  /* current mode: nearest-even */
+                    if (r < -8.0f) r = -8.0f;
+                    if (r > 7.0f) r = 7.0f;
+                    code = (int)r + 8;
+                }
+                uint8_t* byte = &packed[n * (K / 2) + k / 2];
+                if (k % 2 == 0) *byte = (uint8_t)((*byte & 0xF0) | code);
+                else            *byte = (uint8_t)((*byte & 0x0F) | (code << 4));
+            }
+        }
+    }
+    return 0;
+}
+
+/* ---- dequantisation ----------------------------------------------------- */
+
+/* wd[n*K + k] = RNE_bf16( (q - 8) * s[n, k/g] ), as bf16 bits. */
+void oracle_dequant(const uint8_t* packed, const uint16_t* scales,
+                    int64_t N, int64_t K, int64_t g, uint16_t* wd) {
+    int64_t KG = K / g;
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t k = 0; k < K; ++k) {
+            uint8_t b = packed[n * (K / 2) + k / 2];
+            int q = (k % 2 == 0) ? (b & 0x0F) : (b >> 4);
+            float s = oracle_bf16_to_f32(scales[n * KG + k / g]);
+            float prod = (float)(q - 8) * s;  /* exact: 4-bit times 8-bit significand */
+            wd[n * K + k] = oracle_bf16_rne(prod);
+        }
+}
+
+/* ---- linear -------------------------------------------------------------- */
+
+/* One output row: out_row[n] = sum_k x[m,k] * wd[n,k] in fp64, k ascending. */
+static void linear_one_n(const uint16_t* xrow, const uint8_t* packed,
+                         const uint16_t* scales, int64_t n, int64_t K,
+                         int64_t g, double* acc_out) {
+    int64_t KG = K / g;
+    double acc = 0.0;
+    for (int64_t k = 0; k < K; ++k) {
+        uint8_t b = packed[n * (K / 2) + k / 2];
+        int q = (k % 2 == 0) ? (b & 0x0F) : (b >> 4);
+        float s = oracle_bf16_to_f32(scales[n * KG + k / g]);
+        float wd = oracle_bf16_to_f32(oracle_bf16_rne((float)(q - 8) * s));
+        acc += (double)oracle_bf16_to_f32(xrow[k]) * (double)wd;
+    }
+    *acc_out = acc;
+}
+
+/* x: bf16 bits [M, K]; out: fp64 [nrows, N] for the listed rows of x.
+ * nthreads > 1 splits the n loop across OpenMP threads (same arithmetic). */
+void oracle_linear_rows(const uint16_t* x, const uint8_t* packed,
+                        const uint16_t* scales, int64_t M, int64_t N, int64_t K,
+                        int64_t g, const int64_t* rows, int64_t nrows,
+                        double* out, int nthreads) {
+    (void)M;
+    for (int64_t r = 0; r < nrows; ++r) {
+        const uint16_t* xrow = x + rows[r] * K;
+#ifdef _OPENMP
+        #pragma omp parallel for num_threads(nthreads > 0 ? nthreads : 1) schedule(static)
+#endif
+        for (int64_t n = 0; n < N; ++n)
+            linear_one_n(xrow, packed, scales, n, K, g, &out[r * N + n]);
+    }
+    (void)nthreads;
+}
+
+/* Sampled points: out[i] = ref[mi[i], ni[i]]. */
+void oracle_linear_points(const uint16_t* x, const uint8_t* packed,
+                          const uint16_t* scales, int64_t M, int64_t N, int64_t K,
+                          int64_t g, const int64_t* mi, const int64_t* ni,
+                          int64_t npts, double* out, int nthreads) {
+    (void)M; (void)N;
+#ifdef _OPENMP
+    #pragma omp parallel for num_threads(nthreads > 0 ? nthreads : 1) schedule(static)
+#endif
+    for (int64_t i = 0; i < npts; ++i)
+        linear_one_n(x + mi[i] * K, packed, scales, ni[i], K, g, &out[i]);
+    (void)nthreads;
+}
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
