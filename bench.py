@@ -1,0 +1,513 @@
+#!/usr/bin/env python
+"""Benchmark of the W4A16 linear hot path on GB300.
+
+Default step: one pass of the 175B-class int4 linear stack -- 96 layers x
+{QKV 12288->36864, O 12288->12288, up 12288->49152, down 49152->12288},
+g = 128, all ~88 GB of packed weights resident in HBM -- over a batch of 64
+protein-ligand pairs x 1024 tokens (M = 65536).  `value` is scored pairs/s.
+
+Other workloads (--config qkv | mlp_up | mlp_down | gemv | tiny) print the
+same JSON line for one linear (TFLOP/s, or GB/s for the small-M kernel).
+
+--impl reference times the CPU oracle (the only reference there is) on a
+bounded sample of the same workload on the host cores.
+
+Multi-GPU (torchrun): the stack is replicated per GPU and the pairs are
+data-parallel (no collective on the data path); value = pairs of all ranks
+/ max-over-ranks time, scaling "weak".
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "W4A16 GEMM TFLOP/s & % of roofline; scored pairs/s on 175B-class linear stack"
+
+# ncu DRAM traffic (read + write bytes per launch) of the fused kernel, keyed by
+# the hash of the kernel sources the counters were taken on (see profiles/).
+# A mismatch (the kernel changed since) reports traffic as null.
+NCU_TRAFFIC = {}
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_30877_gb300", "csrc")
+    for name in ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def load_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d["bf16_tflops_sustained"], "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+# ----------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        import tempfile
+        fd, self.path = tempfile.mkstemp(prefix="clk_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self) -> dict:
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        def num(s):
+            try:
+                return float(s)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        smax = max(num(r[2]) or 0 for r in rows)
+        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        loaded = [s for s in sm if s >= 0.5 * smax] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": smax,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(power) if power else None}
+
+
+# ----------------------------------------------------------------- distributed
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_dist(world, local):
+    import torch
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return dist if world > 1 else None
+
+
+def barrier(dist):
+    import torch
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+
+def max_over_ranks(dist, v: float) -> float:
+    import torch
+    if dist is None:
+        return v
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------- workloads
+
+def linear_flops(M, N, K):
+    return 2.0 * M * N * K
+
+
+def linear_bytes(M, N, K, g):
+    """Algorithmic bytes of one linear: packed weights + scales + x once + out once."""
+    return N * K / 2 + 2.0 * N * (K // g) + 2.0 * M * K + 2.0 * M * N
+
+
+def make_weights(N, K, g, seed):
+    from paper_2608_30877_gb300 import synthetic as S
+    from paper_2608_30877_gb300 import w4a16 as W
+    w = S.make_w_master(N, K, seed, "cuda")
+    packed, scales = W.quantize(w, g)
+    del w
+    return packed, scales
+
+
+class StackWorkload:
+    def __init__(self, pairs, tokens, layers, g=128):
+        import torch
+        from paper_2608_30877_gb300 import synthetic as S
+        from paper_2608_30877_gb300 import w4a16 as W
+        self.M = pairs * tokens
+        self.pairs = pairs
+        self.layers = layers
+        self.g = g
+        self.flops = 0.0
+        self.bytes = 0.0
+        # one resident activation and output buffer per linear shape
+        self.x = [S.make_x(self.M, K, 2000 + j, "cuda") for j, (_, K, _) in enumerate(S.LAYER_LINEARS)]
+        self.out = [torch.empty((self.M, N), dtype=torch.bfloat16, device="cuda")
+                    for (_, _, N) in S.LAYER_LINEARS]
+        entries = []
+        self.w = []
+        for l in range(layers):
+            for j, (_, K, N) in enumerate(S.LAYER_LINEARS):
+                packed, scales = make_weights(N, K, g, 1000 + 4 * l + j)
+                self.w.append((packed, scales))
+                entries.append((self.x[j], packed, scales, self.out[j]))
+                self.flops += linear_flops(self.M, N, K)
+                self.bytes += linear_bytes(self.M, N, K, g)
+        torch.cuda.synchronize()
+        self.entries = entries
+        self.arr = W.make_layer_array(entries)
+        self.launches_per_step = len(entries)
+
+    def step(self, stream=None):
+        from paper_2608_30877_gb300 import w4a16 as W
+        W.linear_stack_array(self.arr, self.M, self.g, stream)
+
+    def per_linear(self, reps=3):
+        """Event-timed TFLOP/s of each linear shape (layer 0), outside the timed region."""
+        import torch
+        from paper_2608_30877_gb300 import synthetic as S
+        from paper_2608_30877_gb300 import w4a16 as W
+        res = {}
+        for j, (name, K, N) in enumerate(S.LAYER_LINEARS):
+            x, packed, scales, out = self.entries[j]
+            W.linear(x, packed, scales, self.g, out=out)
+            ts = []
+            for _ in range(reps):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                W.linear(x, packed, scales, self.g, out=out)
+                b.record()
+                b.synchronize()
+                ts.append(a.elapsed_time(b) / 1e3)
+            t = statistics.median(ts)
+            res[name] = {"ms": t * 1e3, "tflops": linear_flops(self.M, N, K) / t / 1e12}
+        return res
+
+
+class LinearWorkload:
+    """One linear shape; for the small-M kernel the weights rotate over copies
+    so that no launch finds its weights in L2."""
+
+    def __init__(self, name, M, N, K, g, seed, copies=1):
+        import torch
+        from paper_2608_30877_gb300 import synthetic as S
+        self.name, self.M, self.N, self.K, self.g = name, M, N, K, g
+        self.x = S.make_x(M, K, seed, "cuda")
+        self.out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        self.w = [make_weights(N, K, g, seed + 10 * c) for c in range(copies)]
+        self.flops = linear_flops(M, N, K)
+        self.bytes = linear_bytes(M, N, K, g)
+        self.launches_per_step = 1
+        self.i = 0
+
+    def step(self, stream=None):
+        from paper_2608_30877_gb300 import w4a16 as W
+        packed, scales = self.w[self.i % len(self.w)]
+        self.i += 1
+        W.linear(self.x, packed, scales, self.g, out=self.out, stream=stream)
+
+
+# ----------------------------------------------------------------- CPU oracle
+
+def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 64):
+    """Times the oracle on `r` token rows x N_rows weight rows of one K-deep
+    linear with seeded inputs; grows r until the sample takes ~target_s.
+    Returns (MAC/s, description, threads)."""
+    import numpy as np
+    from oracle import oracle as O
+    from paper_2608_30877_gb300 import synthetic as S
+    w = S.make_w_master(N_rows, K, 1000, "cpu").numpy()
+    packed, scales = O.quantize(w, 128)
+    x = S.bf16_bits(S.make_x(rows_max, K, 2000, "cpu"))
+    threads = len(os.sched_getaffinity(0))
+    r, spent, macs = 1, 0.0, 0
+    while True:
+        t0 = time.perf_counter()
+        O.linear_rows(x[:r], packed, scales, N_rows, K, 128, nthreads=threads)
+        dt = time.perf_counter() - t0
+        spent += dt
+        macs_r = r * N_rows * K
+        if dt >= target_s / 3 or r >= rows_max or spent >= target_s:
+            desc = (f"oracle fp64 linear, {r} token rows x {N_rows} weight rows x K={K} "
+                    f"({macs_r / 1e9:.2f} GMAC) in {dt:.2f} s on {threads} threads")
+            return macs_r / dt, desc, threads
+        r = min(rows_max, max(r + 1, int(r * (target_s / 3) / max(dt, 1e-3))))
+
+
+def stack_macs_per_pair(tokens=1024, layers=96):
+    from paper_2608_30877_gb300 import synthetic as S
+    return tokens * layers * sum(N * K for (_, K, N) in S.LAYER_LINEARS)
+
+
+# ----------------------------------------------------------------- main
+
+def config_for(args):
+    from paper_2608_30877_gb300 import synthetic as S
+    c = args.config
+    if c == "stack":
+        return {"workload": "175B-class int4 linear stack, 96 layers x {qkv 12288->36864, "
+                            "o 12288->12288, up 12288->49152, down 49152->12288}, "
+                            f"M={args.pairs * 1024} ({args.pairs} pairs x 1024 tokens), g=128",
+                "pairs": args.pairs, "tokens_per_pair": 1024, "layers": args.layers, "g": 128,
+                "l2": "inputs larger than L2 (88 GB packed weights, >=1.6 GB activations per "
+                      "linear); no flush"}
+    cases = {"qkv": S.QKV_PREFILL, "mlp_up": S.MLP_UP, "mlp_down": S.MLP_DOWN, "tiny": S.TINY}
+    if c == "gemv":
+        lc = S.gemv_case(args.m)
+    else:
+        lc = cases[c]
+    return {"workload": lc.name, "M": lc.M, "N": lc.N, "K": lc.K, "g": lc.g,
+            "l2": "weights rotate over 2 copies larger than L2" if c == "gemv"
+            else "inputs larger than L2; no flush"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2608_30877_gb300 import synthetic as S
+    if args.config == "stack":
+        K, N_rows = S.D_MODEL, 2048
+        unit = "pairs/s"
+        per_unit = stack_macs_per_pair(1024, args.layers)
+    else:
+        cfg = config_for(args)
+        K, N_rows = cfg["K"], min(cfg["N"], 2048)
+        unit = "TFLOP/s"
+        per_unit = None
+    vals = []
+    desc, threads = "", 1
+    for i in range(args.warmup + args.steps):
+        mac_s, desc, threads = oracle_sample(K, N_rows, target_s=args.ref_seconds)
+        if i >= args.warmup:
+            vals.append(mac_s)
+    mac_s = statistics.median(vals)
+    value = mac_s / per_unit if per_unit else 2 * mac_s / 1e12
+    step_ms = 1e3 * (per_unit / mac_s if per_unit else 0)
+    line = {"metric": METRIC, "impl": "reference", "value": value, "unit": unit, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config_for(args),
+            "cpu_baseline": {"value": value, "unit": unit, "cores": threads, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="stack",
+                    choices=["stack", "qkv", "mlp_up", "mlp_down", "gemv", "tiny"])
+    ap.add_argument("--m", type=int, default=32, help="tokens for --config gemv")
+    ap.add_argument("--pairs", type=int, default=64)
+    ap.add_argument("--layers", type=int, default=96)
+    ap.add_argument("--ref-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dist = init_dist(world, local)
+    from paper_2608_30877_gb300 import w4a16 as W
+    W.lib()
+    peaks = load_peaks()
+
+    setup_t0 = time.perf_counter()
+    if args.config == "stack":
+        wl = StackWorkload(args.pairs, 1024, args.layers)
+        unit = "pairs/s"
+        units_per_step = wl.pairs
+    else:
+        from paper_2608_30877_gb300 import synthetic as S
+        cfg = config_for(args)
+        copies = 2 if args.config == "gemv" else 1
+        wl = LinearWorkload(cfg["workload"], cfg["M"], cfg["N"], cfg["K"], cfg["g"], 3, copies)
+        unit = "GB/s" if args.config == "gemv" else "TFLOP/s"
+        units_per_step = None
+    setup_s = time.perf_counter() - setup_t0
+
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        wl.step()
+    barrier(dist)
+
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device() if "CUDA_VISIBLE_DEVICES" not in os.environ
+                      else local) as clk:
+        barrier(dist)
+        start.record(stream)
+        for _ in range(args.steps):
+            wl.step()
+        end.record(stream)
+        end.synchronize()
+        barrier(dist)
+    elapsed = start.elapsed_time(end) / 1e3
+    elapsed = max_over_ranks(dist, elapsed)
+    step_s = elapsed / args.steps
+    if W.get_device_error() != W.OK:
+        raise RuntimeError("device status word set during the timed region")
+
+    if args.config == "stack":
+        value = world * units_per_step / step_s
+    elif args.config == "gemv":
+        value = world * wl.bytes / step_s / 1e9
+    else:
+        value = world * wl.flops / step_s / 1e12
+
+    # roofline of the fused kernel: every launch in the step is that kernel
+    per_launch_s = step_s / wl.launches_per_step
+    if args.config == "gemv":
+        achieved = wl.bytes / step_s / 1e9
+        peak = peaks["hbm_gbs"]
+        roof = {"bound": "hbm", "unit": "GB/s"}
+    else:
+        achieved = wl.flops / step_s / 1e12
+        peak = peaks["bf16_tflops_sustained"] if args.config == "stack" else peaks["bf16_tflops"]
+        roof = {"bound": "tensor", "unit": "TFLOP/s"}
+    traffic = NCU_TRAFFIC.get((args.config, kernel_source_hash()))
+    roof.update({"achieved": achieved, "peak": peak, "frac": achieved / peak,
+                 "traffic": traffic, "peak_source": peaks["source"] + (
+                     " bf16_tflops_sustained" if args.config == "stack" else
+                     (" hbm_gbs" if args.config == "gemv" else " bf16_tflops")),
+                 "per_launch_ms": per_launch_s * 1e3,
+                 "algorithmic_bytes_per_step": wl.bytes, "flops_per_step": wl.flops})
+
+    line = {"metric": METRIC, "value": value, "unit": unit, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": config_for(args), "clocks": clk.summary(), "roofline": roof,
+            "gpu_launches": wl.launches_per_step * args.steps, "setup_s": setup_s}
+    if args.config == "stack":
+        line["tflops"] = wl.flops / step_s / 1e12
+        if rank == 0:
+            line["per_linear"] = wl.per_linear()
+
+    # end to end through the public API with host buffers
+    if not args.no_e2e:
+        line["e2e"] = e2e(wl, args, dist, world, unit, units_per_step)
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from paper_2608_30877_gb300 import synthetic as S
+        if args.config == "stack":
+            mac_s, desc, threads = oracle_sample(S.D_MODEL, 2048, 15.0)
+            cb = mac_s / stack_macs_per_pair(1024, args.layers)
+            line["cpu_baseline"] = {"value": cb, "unit": "pairs/s", "cores": threads,
+                                    "kind": "oracle", "sample": desc}
+        else:
+            cfg = config_for(args)
+            mac_s, desc, threads = oracle_sample(cfg["K"], min(cfg["N"], 2048), 15.0)
+            if args.config == "gemv":
+                cb = (wl.bytes / (cfg["M"] * cfg["N"] * cfg["K"] / mac_s)) / 1e9
+                cu = "GB/s"
+            else:
+                cb, cu = 2 * mac_s / 1e12, "TFLOP/s"
+            line["cpu_baseline"] = {"value": cb, "unit": cu, "cores": threads,
+                                    "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def e2e(wl, args, dist, world, unit, units_per_step):
+    """Same metric, host buffers: per step the step's inputs are copied from
+    pinned host memory, the library runs, and the result is read back."""
+    import torch
+    if isinstance(wl, StackWorkload):
+        srcs = [torch.empty_like(x, device="cpu").pin_memory() for x in wl.x]
+        for s, x in zip(srcs, wl.x):
+            s.copy_(x)
+        result = wl.out[-1]
+    else:
+        srcs = [torch.empty_like(wl.x, device="cpu").pin_memory()]
+        srcs[0].copy_(wl.x)
+        result = wl.out
+    dsts = wl.x if isinstance(wl, StackWorkload) else [wl.x]
+    host_out = torch.empty_like(result, device="cpu").pin_memory()
+    h2d = sum(s.numel() * s.element_size() for s in srcs)
+    d2h = host_out.numel() * host_out.element_size()
+
+    def one():
+        for s, d in zip(srcs, dsts):
+            d.copy_(s, non_blocking=True)
+        wl.step()
+        host_out.copy_(result, non_blocking=True)
+
+    one()
+    barrier(dist)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = max(1, min(args.steps, 2)) if isinstance(wl, StackWorkload) else args.steps
+    a.record()
+    for _ in range(steps):
+        one()
+    b.record()
+    b.synchronize()
+    t = max_over_ranks(dist, a.elapsed_time(b) / 1e3) / steps
+    if isinstance(wl, StackWorkload):
+        v = world * units_per_step / t
+    elif unit == "GB/s":
+        v = world * wl.bytes / t / 1e9
+    else:
+        v = world * wl.flops / t / 1e12
+    return {"value": v, "unit": unit, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": steps}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,135 @@
+/*
+ * w4a16.h -- C ABI of the GB300 (sm_103a) group-wise int4 weight-only linear
+ * layer library.
+ *
+ * The operation.  The paper scores protein-ligand pairs with a 175B-class
+ * decoder run "4-bit pre-quantized" with "mixed-precision quantization"
+ * (Sec. 3.1, Sec. 4.1), in batches through its prediction module
+ * (Sec. 3.3).  On the prefill path the linear layers (fused QKV, attention
+ * output, MLP up, MLP down) are y = x W^T with W held at 4 bits.  The paper
+ * gives no format; this library fixes one:
+ *
+ *   w_packed  uint8 [N, K/2]   byte (n, j) holds the code of k = 2j in bits
+ *                              0..3 and of k = 2j+1 in bits 4..7; codes are
+ *                              0..15 with zero point 8 (symmetric int4)
+ *   scales    bf16  [N, K/g]   one scale per row n and group of g consecutive k
+ *   dequant   wd[n,k] = RNE_bf16((code - 8) * scales[n, k/g])
+ *   x         bf16  [M, K]     activations (M = packed tokens of the batch)
+ *   out       bf16  [M, N]     out[m,n] = RNE_bf16( sum_k x[m,k] * wd[n,k] ),
+ *                              the sum accumulated in fp32 in an unspecified
+ *                              order
+ *
+ * All matrices are row-major with the last dimension contiguous and no
+ * padding between rows.
+ *
+ * Conventions shared by every entry point:
+ *   - Every buffer is owned by the caller and lives in device memory unless
+ *     stated otherwise.  The library allocates nothing per call, frees
+ *     nothing and does not synchronise: work is enqueued on `stream` and the
+ *     call returns.  `stream` is a cudaStream_t passed as void* (0 = the
+ *     legacy default stream).  `out` must not overlap any input.
+ *   - Arguments are validated before anything is launched; a rejected call
+ *     launches nothing and leaves every buffer untouched.
+ *   - Device pointers must be 16-byte aligned (W4A16_ERR_ALIGNMENT).
+ *   - Supported shapes: M, N >= 1; K >= g; g a multiple of 64; K a multiple
+ *     of g; M, N, K < 2^31 (W4A16_ERR_INVALID_ARG / W4A16_ERR_UNSUPPORTED).
+ *     g = 128 is the tuned case.
+ *   - A launch failure returns W4A16_ERR_CUDA (the CUDA error is left for
+ *     cudaGetLastError to report).
+ *   - The kernels bound every internal wait.  If a wait runs out (it never
+ *     should) the kernel records W4A16_ERR_TIMEOUT in a device status word
+ *     and finishes early; w4a16_get_device_error reports it.
+ *   - Results are deterministic: the same inputs give the same bits.
+ *   - Thread safety: calls from several host threads are safe; per-device
+ *     state (SM count, driver entry point) is initialised once.
+ */
+#ifndef W4A16_H
+#define W4A16_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    W4A16_OK = 0,
+    W4A16_ERR_INVALID_ARG = 1,   /* null pointer, non-positive or inconsistent size */
+    W4A16_ERR_UNSUPPORTED = 2,   /* valid request outside the supported shapes */
+    W4A16_ERR_ALIGNMENT = 3,     /* a pointer is not 16-byte aligned */
+    W4A16_ERR_CUDA = 4,          /* a CUDA runtime/driver call or launch failed */
+    W4A16_ERR_TIMEOUT = 5        /* a kernel gave up on a bounded wait */
+} w4a16_status;
+
+/*
+ * out = x * dequant(w_packed, scales)^T.
+ * The hot path of the paper's scoring workflow (Sec. 3.3: batched encoding and
+ * affinity prediction) for one int4 linear layer (Sec. 3.1, Sec. 4.1).
+ *   x_bf16       [M, K]   bf16, device
+ *   w_packed_u8  [N, K/2] uint8, device, layout above
+ *   scales_bf16  [N, K/g] bf16, device
+ *   out_bf16     [M, N]   bf16, device, written in full
+ * M <= 32 runs the bandwidth-bound small-M kernel, larger M the tensor-core
+ * GEMM; both are the same fused dequant + tcgen05 MMA design.
+ */
+int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
+                 void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,
+                 void* stream);
+
+/* One int4 linear layer of a stack.  The caller owns every pointer. */
+typedef struct {
+    const void* x;          /* bf16 [M, K] */
+    const void* w_packed;   /* uint8 [N, K/2] */
+    const void* scales;     /* bf16 [N, K/g] */
+    void* out;              /* bf16 [M, N] */
+    int64_t N;
+    int64_t K;
+} w4a16_layer;
+
+/*
+ * Runs n_layers linear layers in order on `stream`, all with the same M
+ * (packed tokens of the scored batch) and group size g: the per-pass layer
+ * loop of the paper's prediction module (Sec. 3.3) over the quantised
+ * decoder (Sec. 4.1).  `layers` is a HOST array the call reads before it
+ * returns.  Every layer is validated before the first launch; layer i may read
+ * the output of layer i-1 (chaining) because launches are stream-ordered.
+ */
+int w4a16_linear_stack(const w4a16_layer* layers, int64_t n_layers,
+                       int64_t M, int64_t g, void* stream);
+
+/*
+ * wd = dequant(w_packed, scales) as bf16 [N, K] (device).  The same unpack
+ * and rounding as inside the GEMM, exported so that it can be compared bit
+ * for bit with the definition above.
+ */
+int w4a16_dequant(const void* w_packed_u8, const void* scales_bf16, void* w_bf16,
+                  int64_t N, int64_t K, int64_t g, void* stream);
+
+/*
+ * Quantises fp32 master weights w_f32 [N, K] (device) into w_packed_u8 and
+ * scales_bf16 with the library's format: per (n, group), s = RNE_bf16(amax/7)
+ * with an IEEE fp32 division, code = clamp(round_half_even(w/s), -8, 7) + 8,
+ * an all-zero group gets s = 0 and code 8.  Weight preparation, not part of
+ * the per-token path.
+ */
+int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales_bf16,
+                   int64_t N, int64_t K, int64_t g, void* stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the device status word that
+ * kernels set when a bounded wait runs out.  Returns W4A16_OK,
+ * W4A16_ERR_TIMEOUT or W4A16_ERR_CUDA.
+ */
+int w4a16_get_device_error(void* stream);
+
+/* Static text for a status code; never NULL. */
+const char* w4a16_status_string(int status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int w4a16_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* W4A16_H */

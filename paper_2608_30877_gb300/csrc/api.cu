@@ -1,0 +1,254 @@
+// C ABI of the library (declared in include/w4a16.h): argument validation,
+// TMA descriptor encoding, kernel dispatch and the device status word.
+#include "internal.h"
+#include "w4a16.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <cstdlib>
+#include <mutex>
+
+namespace w4a16 {
+namespace {
+
+// Set by kernels when a bounded wait runs out; read and cleared by
+// w4a16_get_device_error.
+__device__ int g_status_word;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+    bool ready = false;
+    int sm_count = 0;
+    int* status = nullptr;
+};
+
+std::mutex g_mutex;
+DeviceState g_dev[kMaxDevices];
+EncodeTiledFn g_encode = nullptr;
+int g_group_t = 8;
+
+// Per-device set-up, done once with the device current.
+int device_state(DeviceState** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return W4A16_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mutex);
+    DeviceState& st = g_dev[dev];
+    if (!st.ready) {
+        if (g_encode == nullptr) {
+            void* fn = nullptr;
+            cudaDriverEntryPointQueryResult q;
+            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                 cudaEnableDefault, &q) != cudaSuccess ||
+                q != cudaDriverEntryPointSuccess || fn == nullptr)
+                return W4A16_ERR_CUDA;
+            g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+            if (const char* e = std::getenv("W4A16_GROUP_T")) {
+                const int v = std::atoi(e);
+                if (v > 0 && v <= 4096) g_group_t = v;
+            }
+        }
+        if (cudaDeviceGetAttribute(&st.sm_count, cudaDevAttrMultiProcessorCount, dev) !=
+            cudaSuccess)
+            return W4A16_ERR_CUDA;
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return W4A16_ERR_CUDA;
+        st.status = static_cast<int*>(p);
+        st.ready = true;
+    }
+    *out = &st;
+    return W4A16_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlaps(const void* a, int64_t na, const void* b, int64_t nb) {
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+    return a0 < b0 + static_cast<uintptr_t>(nb) && b0 < a0 + static_cast<uintptr_t>(na);
+}
+
+constexpr int64_t kMaxDim = (int64_t{1} << 31) - 1;
+
+int check_weights(const void* w, const void* s, int64_t N, int64_t K, int64_t g) {
+    if (w == nullptr || s == nullptr) return W4A16_ERR_INVALID_ARG;
+    if (N <= 0 || K <= 0 || g <= 0) return W4A16_ERR_INVALID_ARG;
+    if (K % g != 0) return W4A16_ERR_INVALID_ARG;
+    if (g % 64 != 0) return W4A16_ERR_UNSUPPORTED;
+    if (N > kMaxDim || K > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(w) || !aligned16(s)) return W4A16_ERR_ALIGNMENT;
+    return W4A16_OK;
+}
+
+int check_linear(const void* x, const void* w, const void* s, const void* out, int64_t M,
+                 int64_t N, int64_t K, int64_t g) {
+    if (x == nullptr || out == nullptr) return W4A16_ERR_INVALID_ARG;
+    if (M <= 0) return W4A16_ERR_INVALID_ARG;
+    const int rc = check_weights(w, s, N, K, g);
+    if (rc != W4A16_OK) return rc;
+    if (M > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(x) || !aligned16(out)) return W4A16_ERR_ALIGNMENT;
+    const int64_t out_bytes = M * N * 2;
+    if (overlaps(out, out_bytes, x, M * K * 2) || overlaps(out, out_bytes, w, N * (K / 2)) ||
+        overlaps(out, out_bytes, s, N * (K / g) * 2))
+        return W4A16_ERR_INVALID_ARG;
+    // tile counts must fit the kernel's int arithmetic
+    const int64_t tiles = ((M + 31) / 32) * ((N + 127) / 128);
+    if (tiles > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    return W4A16_OK;
+}
+
+int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uint64_t inner,
+              uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
+              CUtensorMapSwizzle swz) {
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = g_encode(map, dtype, 2, const_cast<void*>(base), dims, strides, box, estr,
+                                CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? W4A16_OK : W4A16_ERR_CUDA;
+}
+
+// Validated arguments -> one kernel launch.
+int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
+                  int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
+    const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
+    const int T = ts_tokens_per_tile(v);
+    alignas(64) CUtensorMap tx;
+    alignas(64) CUtensorMap tw;
+    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
+                       CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != W4A16_OK) return rc;
+    rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 32, 128,
+                   CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (rc != W4A16_OK) return rc;
+    TsParams p;
+    p.scales = static_cast<const uint16_t*>(s);
+    p.out = static_cast<uint16_t*>(out);
+    p.status = st.status;
+    p.M = static_cast<int>(M);
+    p.N = static_cast<int>(N);
+    p.K = static_cast<int>(K);
+    p.g = static_cast<int>(g);
+    p.num_t_tiles = static_cast<int>((M + T - 1) / T);
+    p.num_w_tiles = static_cast<int>((N + 127) / 128);
+    p.num_tiles = p.num_t_tiles * p.num_w_tiles;
+    p.group_t = v == TsVariant::kGemm256 ? g_group_t : 1;
+    const int grid = ts_grid(v, p, st.sm_count);
+    return ts_launch(v, &tx, &tw, p, grid, stream) == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace w4a16
+
+using namespace w4a16;
+
+extern "C" int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
+                            void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,
+                            void* stream) {
+    int rc = check_linear(x_bf16, w_packed_u8, scales_bf16, out_bf16, M, N, K, g);
+    if (rc != W4A16_OK) return rc;
+    DeviceState* st = nullptr;
+    rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    return launch_linear(*st, x_bf16, w_packed_u8, scales_bf16, out_bf16, M, N, K, g,
+                         static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int w4a16_linear_stack(const w4a16_layer* layers, int64_t n_layers, int64_t M,
+                                  int64_t g, void* stream) {
+    if (layers == nullptr || n_layers <= 0) return W4A16_ERR_INVALID_ARG;
+    for (int64_t i = 0; i < n_layers; ++i) {
+        const w4a16_layer& l = layers[i];
+        const int rc = check_linear(l.x, l.w_packed, l.scales, l.out, M, l.N, l.K, g);
+        if (rc != W4A16_OK) return rc;
+    }
+    DeviceState* st = nullptr;
+    int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    for (int64_t i = 0; i < n_layers; ++i) {
+        const w4a16_layer& l = layers[i];
+        rc = launch_linear(*st, l.x, l.w_packed, l.scales, l.out, M, l.N, l.K, g,
+                           static_cast<cudaStream_t>(stream));
+        if (rc != W4A16_OK) return rc;
+    }
+    return W4A16_OK;
+}
+
+extern "C" int w4a16_dequant(const void* w_packed_u8, const void* scales_bf16, void* w_bf16,
+                             int64_t N, int64_t K, int64_t g, void* stream) {
+    int rc = check_weights(w_packed_u8, scales_bf16, N, K, g);
+    if (rc != W4A16_OK) return rc;
+    if (w_bf16 == nullptr) return W4A16_ERR_INVALID_ARG;
+    if (!aligned16(w_bf16)) return W4A16_ERR_ALIGNMENT;
+    if (overlaps(w_bf16, N * K * 2, w_packed_u8, N * (K / 2)) ||
+        overlaps(w_bf16, N * K * 2, scales_bf16, N * (K / g) * 2))
+        return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    return launch_dequant(static_cast<const uint8_t*>(w_packed_u8),
+                          static_cast<const uint16_t*>(scales_bf16),
+                          static_cast<uint16_t*>(w_bf16), N, K, g,
+                          static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales_bf16, int64_t N,
+                              int64_t K, int64_t g, void* stream) {
+    int rc = check_weights(w_packed_u8, scales_bf16, N, K, g);
+    if (rc != W4A16_OK) return rc;
+    if (w_f32 == nullptr) return W4A16_ERR_INVALID_ARG;
+    if (!aligned16(w_f32)) return W4A16_ERR_ALIGNMENT;
+    if (overlaps(w_f32, N * K * 4, w_packed_u8, N * (K / 2)) ||
+        overlaps(w_f32, N * K * 4, scales_bf16, N * (K / g) * 2) ||
+        overlaps(w_packed_u8, N * (K / 2), scales_bf16, N * (K / g) * 2))
+        return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    return launch_quantize(static_cast<const float*>(w_f32), static_cast<uint8_t*>(w_packed_u8),
+                           static_cast<uint16_t*>(scales_bf16), N, K, g,
+                           static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_get_device_error(void* stream) {
+    DeviceState* st = nullptr;
+    int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return W4A16_ERR_CUDA;
+    int v = 0;
+    const int zero = 0;
+    if (cudaMemcpy(&v, st->status, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemcpy(st->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
+        return W4A16_ERR_CUDA;
+    return v == 0 ? W4A16_OK : v;
+}
+
+extern "C" const char* w4a16_status_string(int status) {
+    switch (status) {
+        case W4A16_OK: return "ok";
+        case W4A16_ERR_INVALID_ARG: return "invalid argument";
+        case W4A16_ERR_UNSUPPORTED: return "unsupported shape or group size";
+        case W4A16_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
+        case W4A16_ERR_CUDA: return "CUDA error";
+        case W4A16_ERR_TIMEOUT: return "kernel wait timed out";
+        default: return "unknown status";
+    }
+}
+
+extern "C" int w4a16_version(void) { return 100; }

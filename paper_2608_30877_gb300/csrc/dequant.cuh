@@ -1,0 +1,56 @@
+// Register-level int4 -> bf16 dequantisation shared by every kernel of the
+// library (the exported dequant, the GEMM and the small-M path), so that the
+// GEMM's weights are bit-identical to w4a16_dequant's output.
+//
+// A packed 32-bit word holds eight consecutive codes q_0..q_7 of one row
+// (q_i in bits 4i..4i+3: byte j carries the even k in its low nibble and the
+// odd k in its high nibble).  For each pair (q_2j, q_2j+1) the word is turned
+// into a bf16x2 without any int->float conversion:
+//   - PRMT puts byte j of w in byte 0 and byte j of (w >> 4) in byte 2;
+//   - masking to bits 0..3 / 16..19 and OR-ing 0x4300 into each half gives
+//     the bf16 pattern 0x430q, whose value is 128 + q (bf16 spacing on
+//     [128, 256) is exactly 1);
+//   - a bf16x2 subtraction of 136 gives q - 8 exactly (|q - 8| <= 8);
+//   - a bf16x2 multiply by the scale rounds the exact product once, to
+//     nearest even -- the definition wd = RNE_bf16((q - 8) * s).
+#pragma once
+
+#include <cstdint>
+
+namespace w4a16 {
+
+__device__ __forceinline__ uint32_t prmt_b32(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t bf16x2_sub(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t bf16x2_mul(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+
+// 8 codes -> 4 bf16x2 words; out[j] = (wd(k=2j) low half, wd(k=2j+1) high half).
+// s2 holds the row's bf16 scale in both halves.
+__device__ __forceinline__ void dequant_word(uint32_t w, uint32_t s2, uint32_t* out) {
+    const uint32_t w4 = w >> 4;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        uint32_t t = prmt_b32(w, w4, static_cast<uint32_t>(j | ((4 + j) << 8)));
+        t = (t & 0x000F000Fu) | 0x43004300u;               // (128 + q_2j, 128 + q_2j+1)
+        out[j] = bf16x2_mul(bf16x2_sub(t, 0x43084308u), s2);  // (q - 8) * s, one rounding
+    }
+}
+
+__device__ __forceinline__ uint32_t splat_bf16(uint16_t s) {
+    return static_cast<uint32_t>(s) | (static_cast<uint32_t>(s) << 16);
+}
+
+}  // namespace w4a16

@@ -1,0 +1,42 @@
+// Internal interface between the C-ABI layer (api.cu) and the kernel
+// translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace w4a16 {
+
+// Parameters of the fused dequant + tcgen05 kernel (everything except the
+// two TMA descriptors, which are passed as __grid_constant__ arguments).
+struct TsParams {
+    const uint16_t* scales;  // bf16 bits [N, K/g]
+    uint16_t* out;           // bf16 bits [M, N]
+    int* status;             // device status word (timeouts)
+    int M, N, K, g;
+    int num_t_tiles;         // token tiles:  ceil(M / tokens per tile)
+    int num_w_tiles;         // weight tiles: ceil(N / 128)
+    int num_tiles;
+    int group_t;             // raster: token tiles per group
+};
+
+// Kernel variants of the fused kernel.  Both take 128 weight rows per tile
+// (the MMA's M) and 64 k per pipeline stage.
+enum class TsVariant : int {
+    kGemm256 = 0,  // 256 tokens per tile, persistent grid (large M)
+    kGemv32 = 1,   // 32 tokens per tile, one tile per CTA (M <= 32)
+};
+
+int ts_tokens_per_tile(TsVariant v);
+// Fills the grid size to use for the given problem (persistent or not).
+int ts_grid(TsVariant v, const TsParams& p, int sm_count);
+cudaError_t ts_launch(TsVariant v, const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
+                      const TsParams& p, int grid, cudaStream_t stream);
+
+cudaError_t launch_dequant(const uint8_t* w, const uint16_t* scales, uint16_t* wd, int64_t N,
+                           int64_t K, int64_t g, cudaStream_t stream);
+cudaError_t launch_quantize(const float* w, uint8_t* packed, uint16_t* scales, int64_t N,
+                            int64_t K, int64_t g, cudaStream_t stream);
+
+}  // namespace w4a16

@@ -1,0 +1,365 @@
+// Fused int4-dequant + tcgen05 GEMM for sm_103a.
+//
+// out[m, n] = sum_k x[m, k] * wd[n, k], wd = RNE_bf16((code - 8) * scale).
+//
+// Mapping onto the 5th-generation tensor core.  The MMA computes
+// D[128 x T] = A[128 x 16] * B[T x 16]^T per instruction with
+//   A = 128 dequantised weight rows, held in TENSOR MEMORY,
+//   B = T tokens of x, K-major in shared memory (TMA, 128-byte swizzle),
+//   D = fp32 accumulator in tensor memory: lane = weight row, column = token.
+// Putting the weights in A lets the dequantising warps write bf16 pairs
+// straight from registers into tensor memory (tcgen05.st) -- the 4x larger
+// bf16 weight tile never touches shared memory, which keeps shared-memory
+// bandwidth for the x tiles the MMA reads.
+//
+// Warp roles (320 threads):
+//   warp 0      TMA producer: x tile [T x 64] and packed weight tile [128 x 32 B]
+//               per stage into a ring of S_SMEM shared-memory stages;
+//   warp 1      allocates tensor memory, one thread issues the MMAs;
+//   warps 2..5  dequantisers: thread = one weight row (its TMEM lane),
+//               32 packed bytes -> 64 bf16 -> 32 TMEM columns per stage,
+//               into a ring of S_TMEM tensor-memory A stages;
+//   warps 6..9  epilogue: tcgen05.ld of the accumulator, fp32 -> bf16,
+//               stores to out.
+// A warp may only touch the 32 TMEM lanes of its sub-partition (warp % 4), so
+// each group of four warps covers all 128 lanes.
+//
+// Every wait is bounded (see ptx.cuh); on a timeout the kernel records
+// W4A16_ERR_TIMEOUT, drains its own copies and MMAs, frees tensor memory and
+// returns.
+#include "dequant.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace w4a16 {
+
+namespace {
+
+constexpr int kThreads = 320;
+constexpr int kRows = 128;  // weight rows per tile (MMA M)
+constexpr int kBK = 64;     // k per stage (one 128-byte swizzle row of bf16)
+
+template <int T, int S_SMEM, int S_TMEM>
+struct Layout {
+    static constexpr int X_BYTES = T * kBK * 2;
+    static constexpr int W_BYTES = kRows * kBK / 2;
+    static constexpr int X_OFF = 0;
+    static constexpr int W_OFF = S_SMEM * X_BYTES;
+    static constexpr int BAR_OFF = W_OFF + S_SMEM * W_BYTES;
+    // full_tma[S_SMEM], empty_smem[S_SMEM], full_a[S_TMEM], empty_a[S_TMEM],
+    // d_full, d_empty, drain
+    static constexpr int NBARS = 2 * S_SMEM + 2 * S_TMEM + 3;
+    static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
+    static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;  // + slack for 1024-B alignment
+    static constexpr int D_COL = 0;
+    static constexpr int A_COL = T;
+    static constexpr int COLS_USED = T + S_TMEM * (kBK / 2);
+    static constexpr int TMEM_COLS = COLS_USED <= 32    ? 32
+                                     : COLS_USED <= 64  ? 64
+                                     : COLS_USED <= 128 ? 128
+                                     : COLS_USED <= 256 ? 256
+                                                        : 512;
+    static_assert(COLS_USED <= 512, "tensor memory holds 512 columns");
+    static_assert(X_BYTES % 1024 == 0, "x stages must keep 1024-byte alignment");
+    static_assert(T % 32 == 0 && T >= 32 && T <= 256, "tokens per tile");
+};
+
+__device__ __forceinline__ void tile_coords(int tile, const TsParams& p, int& tt, int& wt) {
+    const int per_group = p.group_t * p.num_w_tiles;
+    const int grp = tile / per_group;
+    const int first_t = grp * p.group_t;
+    const int rest = p.num_t_tiles - first_t;
+    const int gsize = rest < p.group_t ? rest : p.group_t;
+    const int local = tile - grp * per_group;
+    tt = first_t + local % gsize;
+    wt = local / gsize;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+template <int T, int S_SMEM, int S_TMEM, int MIN_BLOCKS>
+__global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
+    w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
+                    const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
+    using L = Layout<T, S_SMEM, S_TMEM>;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t sbase = (raw + 1023u) & ~1023u;
+    uint8_t* smem = smem_raw + (sbase - raw);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    const uint32_t bars = sbase + L::BAR_OFF;
+    auto full_tma = [&](int s) { return bars + 8u * s; };
+    auto empty_smem = [&](int s) { return bars + 8u * (S_SMEM + s); };
+    auto full_a = [&](int s) { return bars + 8u * (2 * S_SMEM + s); };
+    auto empty_a = [&](int s) { return bars + 8u * (2 * S_SMEM + S_TMEM + s); };
+    const uint32_t d_full = bars + 8u * (2 * S_SMEM + 2 * S_TMEM);
+    const uint32_t d_empty = d_full + 8u;
+    const uint32_t drain = d_full + 16u;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S_SMEM; ++s) {
+            mbar_init(full_tma(s), 1);
+            mbar_init(empty_smem(s), 1);
+        }
+        for (int s = 0; s < S_TMEM; ++s) {
+            mbar_init(full_a(s), 4);  // one arrival per dequant warp
+            mbar_init(empty_a(s), 1);
+        }
+        mbar_init(d_full, 1);
+        mbar_init(d_empty, 4);  // one arrival per epilogue warp
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap_x);
+        prefetch_tmap(&tmap_w);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const int KT = p.K / kBK;
+    const int KG = p.K / p.g;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            uint32_t it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+                int tt, wt;
+                tile_coords(tile, p, tt, wt);
+                const int t0 = tt * T, n0 = wt * kRows;
+                for (int kt = 0; kt < KT; ++kt, ++it) {
+                    const int s = it % S_SMEM;
+                    const uint32_t ph = (it / S_SMEM) & 1u;
+                    if (!wait_one(empty_smem(s), ph ^ 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(full_tma(s), L::X_BYTES + L::W_BYTES);
+                    tma_load_2d(sbase + L::X_OFF + s * L::X_BYTES, &tmap_x, full_tma(s), kt * kBK,
+                                t0);
+                    tma_load_2d(sbase + L::W_OFF + s * L::W_BYTES, &tmap_w, full_tma(s),
+                                kt * (kBK / 2), n0);
+                }
+            }
+            // Drain: every load this thread issued has landed before exit.
+            const uint32_t last = it < static_cast<uint32_t>(S_SMEM) ? it : S_SMEM;
+            for (uint32_t i = it - last; i < it; ++i) {
+                uint64_t t0 = global_timer_ns();
+                while (!mbar_try_wait(full_tma(i % S_SMEM), (i / S_SMEM) & 1u)) {
+                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_f32(kRows, T);
+            uint32_t it = 0, tcount = 0;
+            bool ok = true;
+            bool issued = false;
+            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++tcount) {
+                if (!wait_one(d_empty, (tcount & 1u) ^ 1u, abort_flag, p.status)) break;
+                tc_fence_after();
+                for (int kt = 0; kt < KT; ++kt, ++it) {
+                    const int s = it % S_SMEM;
+                    const int sa = it % S_TMEM;
+                    if (!wait_one(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status) ||
+                        !wait_one(full_a(sa), (it / S_TMEM) & 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t xs = sbase + L::X_OFF + s * L::X_BYTES;
+#pragma unroll
+                    for (int ks = 0; ks < kBK / 16; ++ks) {
+                        const uint32_t a = tmem + L::A_COL + sa * (kBK / 2) + ks * 8;
+                        const uint64_t b = sdesc_kmajor_sw128(xs + ks * 32);
+                        tc_mma_ts(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
+                    }
+                    issued = true;
+                    tc_commit(empty_smem(s));
+                    tc_commit(empty_a(sa));
+                }
+                if (!ok) break;
+                tc_commit(d_full);
+            }
+            if (issued) {
+                // Drain: all MMAs issued by this thread have completed.
+                tc_commit(drain);
+                uint64_t t0 = global_timer_ns();
+                while (!mbar_try_wait(drain, 0)) {
+                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
+                }
+            }
+        }
+    } else if (warp < 6) {
+        // ------------------------------------------------------------ dequantisers
+        const int sub = warp & 3;
+        const int r = sub * 32 + lane;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
+        uint32_t it = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+            int tt, wt;
+            tile_coords(tile, p, tt, wt);
+            const int n = wt * kRows + r;
+            const bool valid = n < p.N;
+            const uint16_t* srow = p.scales + static_cast<int64_t>(valid ? n : 0) * KG;
+            uint16_t s_cur = valid ? __ldg(srow) : 0;
+            uint16_t s_nxt = (valid && KG > 1) ? __ldg(srow + 1) : 0;
+            int cur_grp = 0;
+            for (int kt = 0; kt < KT; ++kt, ++it) {
+                const int grp = (kt * kBK) / p.g;
+                if (grp != cur_grp) {
+                    s_cur = s_nxt;
+                    cur_grp = grp;
+                    s_nxt = (valid && grp + 1 < KG) ? __ldg(srow + grp + 1) : 0;
+                }
+                const int s = it % S_SMEM;
+                const int sa = it % S_TMEM;
+                if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status) ||
+                    !wait_warp(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint4* wrow =
+                    reinterpret_cast<const uint4*>(smem + L::W_OFF + s * L::W_BYTES + r * 32);
+                const uint4 w0 = wrow[0];
+                const uint4 w1 = wrow[1];
+                const uint32_t s2 = splat_bf16(s_cur);
+                uint32_t v[32];
+                dequant_word(w0.x, s2, v + 0);
+                dequant_word(w0.y, s2, v + 4);
+                dequant_word(w0.z, s2, v + 8);
+                dequant_word(w0.w, s2, v + 12);
+                dequant_word(w1.x, s2, v + 16);
+                dequant_word(w1.y, s2, v + 20);
+                dequant_word(w1.z, s2, v + 24);
+                dequant_word(w1.w, s2, v + 28);
+                tmem_st_32x32b_x32(lane_base + L::A_COL + sa * (kBK / 2), v);
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(full_a(sa));
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int sub = warp & 3;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
+        const bool n_even = (p.N & 1) == 0;
+        uint32_t tcount = 0;
+        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++tcount) {
+            int tt, wt;
+            tile_coords(tile, p, tt, wt);
+            if (!wait_warp(d_full, tcount & 1u, abort_flag, p.status)) break;
+            tc_fence_after();
+            const int n = wt * kRows + sub * 32 + lane;
+#pragma unroll 1
+            for (int c = 0; c < T / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(lane_base + L::D_COL + c * 32, v);
+                tmem_ld_wait(v);
+                const int mbase = tt * T + c * 32;
+                if (n_even) {
+                    // Pair neighbouring lanes so that each store writes two
+                    // adjacent outputs (n, n+1) of one token as a 32-bit word.
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float f0 = __uint_as_float(v[2 * j]);
+                        const float f1 = __uint_as_float(v[2 * j + 1]);
+                        const float send = (lane & 1) ? f0 : f1;
+                        const float other = __shfl_xor_sync(0xffffffffu, send, 1);
+                        int m, col;
+                        uint32_t word;
+                        if ((lane & 1) == 0) {
+                            m = mbase + 2 * j;
+                            col = n;
+                            word = pack_bf16x2(f0, other);
+                        } else {
+                            m = mbase + 2 * j + 1;
+                            col = n - 1;
+                            word = pack_bf16x2(other, f1);
+                        }
+                        if (m < p.M && col < p.N)
+                            *reinterpret_cast<uint32_t*>(p.out + static_cast<int64_t>(m) * p.N +
+                                                         col) = word;
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int m = mbase + j;
+                        if (m < p.M && n < p.N) {
+                            const uint32_t word = pack_bf16x2(__uint_as_float(v[j]), 0.0f);
+                            p.out[static_cast<int64_t>(m) * p.N + n] =
+                                static_cast<uint16_t>(word & 0xFFFFu);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(d_empty);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
+}
+
+template <int T, int S_SMEM, int S_TMEM, int MIN_BLOCKS>
+cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
+                           int grid, cudaStream_t stream) {
+    using L = Layout<T, S_SMEM, S_TMEM>;
+    auto kern = w4a16_ts_kernel<T, S_SMEM, S_TMEM, MIN_BLOCKS>;
+    // Idempotent; cheap enough to repeat per launch and per device.
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    return cudaGetLastError();
+}
+
+// Large M: 256 tokens per tile, 6 stages of (32 KB x + 4 KB packed weights),
+// tensor memory = 256 accumulator columns + 6 x 32 A columns.
+constexpr int kGemmT = 256, kGemmSS = 6, kGemmST = 6;
+// Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
+// 128 tensor-memory columns so that three CTAs share an SM.
+constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3;
+
+}  // namespace
+
+int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemm256 ? kGemmT : kGemvT; }
+
+int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
+    if (v == TsVariant::kGemm256) return p.num_tiles < sm_count ? p.num_tiles : sm_count;
+    return p.num_tiles;
+}
+
+cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
+                      const TsParams& p, int grid, cudaStream_t stream) {
+    if (v == TsVariant::kGemm256)
+        return launch_variant<kGemmT, kGemmSS, kGemmST, 1>(tx, tw, p, grid, stream);
+    return launch_variant<kGemvT, kGemvSS, kGemvST, 3>(tx, tw, p, grid, stream);
+}
+
+}  // namespace w4a16

@@ -1,0 +1,68 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads, exports
+every function include/w4a16.h declares, and rejects bad arguments before
+touching the device."""
+import ctypes
+
+import pytest
+
+from paper_2608_30877_gb300 import w4a16 as W
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2608_30877_gb300 import build as B
+    B.build()
+    return W.lib()
+
+
+def test_header_declares_the_boundary():
+    names = W.header_functions()
+    for f in ("w4a16_linear", "w4a16_linear_stack", "w4a16_dequant", "w4a16_quantize",
+              "w4a16_get_device_error", "w4a16_status_string", "w4a16_version"):
+        assert f in names
+
+
+def test_every_declared_symbol_is_exported(L):
+    for name in W.header_functions():
+        assert hasattr(L, name), name
+
+
+def test_status_strings(L):
+    assert W.status_string(0) == "ok"
+    assert "aligned" in W.status_string(W.ERR_ALIGNMENT)
+    assert W.status_string(99) == "unknown status"
+    assert W.version() >= 100
+
+
+A = 1 << 20  # fake, 16-byte aligned, non-overlapping "device" addresses (never dereferenced)
+
+
+@pytest.mark.parametrize("args,want", [
+    ((0, A, 2 * A, 3 * A, 4, 8, 256, 128), W.ERR_INVALID_ARG),        # null x
+    ((A, 2 * A, 3 * A, 4 * A, 0, 8, 256, 128), W.ERR_INVALID_ARG),     # M = 0
+    ((A, 2 * A, 3 * A, 4 * A, 4, -1, 256, 128), W.ERR_INVALID_ARG),    # N < 0
+    ((A, 2 * A, 3 * A, 4 * A, 4, 8, 200, 128), W.ERR_INVALID_ARG),     # K % g
+    ((A, 2 * A, 3 * A, 4 * A, 4, 8, 256, 32), W.ERR_UNSUPPORTED),      # g % 64
+    ((A + 8, 2 * A, 3 * A, 4 * A, 4, 8, 256, 128), W.ERR_ALIGNMENT),   # misaligned x
+    ((A, 2 * A, 3 * A, 4 * A + 2, 4, 8, 256, 128), W.ERR_ALIGNMENT),   # misaligned out
+    ((A, 2 * A, 3 * A, A + 64, 4, 8, 256, 128), W.ERR_INVALID_ARG),    # out overlaps x
+    ((A, 2 * A, 3 * A, 4 * A, 1 << 31, 8, 256, 128), W.ERR_UNSUPPORTED),
+])
+def test_linear_rejects_before_launch(L, args, want):
+    assert L.w4a16_linear(*args, None) == want
+
+
+def test_stack_validates_every_layer_first(L):
+    good = W.Layer(A, 2 * A, 3 * A, 4 * A, 8, 256)
+    bad = W.Layer(A, 2 * A, 3 * A, 4 * A, 8, 200)
+    arr = (W.Layer * 2)(good, bad)
+    assert L.w4a16_linear_stack(arr, 2, 4, 128, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_linear_stack(arr, 0, 4, 128, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_linear_stack(None, 1, 4, 128, None) == W.ERR_INVALID_ARG
+
+
+def test_dequant_and_quantize_reject_bad_args(L):
+    assert L.w4a16_dequant(A, 2 * A, 0, 8, 256, 128, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_dequant(A, 2 * A, 3 * A + 4, 8, 256, 128, None) == W.ERR_ALIGNMENT
+    assert L.w4a16_quantize(0, 2 * A, 3 * A, 8, 256, 128, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_quantize(A, 2 * A, 3 * A, 8, 256, 48, None) == W.ERR_INVALID_ARG

@@ -1,0 +1,180 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on
+the same seeded inputs.  Integer work (unpack, dequant, quantise) must be
+bit-exact; linear outputs must satisfy max|gpu-ref| <= 2e-2 * rms(ref) and
+||gpu-ref||_F / ||ref||_F <= 5e-3 per output matrix."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2608_30877_gb300 import synthetic as S
+from tests.gpu_helpers import assert_close, bf16_to_f64, host_case, to_device
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_30877_gb300 import w4a16 as W
+    W.lib()
+    yield
+    assert W.get_device_error() == W.OK
+
+
+def _W():
+    from paper_2608_30877_gb300 import w4a16 as W
+    return W
+
+
+# ---------------------------------------------------------------- dequant
+
+@pytest.mark.parametrize("N,K,g", [(1024, 512, 128), (3, 64, 64), (257, 768, 256), (130, 1024, 128)])
+def test_dequant_bit_exact(N, K, g):
+    W = _W()
+    _, _, packed, scales = host_case(1, N, K, g, 100 + N, 0)
+    want = O.dequant(packed, scales, N, K, g)
+    _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
+    got = W.dequant(wd, sd, g)
+    torch.cuda.synchronize()
+    got = got.cpu().view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(got, want)
+
+
+def test_dequant_every_code_and_rounding_case():
+    W = _W()
+    scales_f = [1.0, 1.0 + 2 ** -7, 0.0078125, 0.10009765625, 3.0, -0.5, 0.0,
+                0.0014982223510742188, 0.02099609375, 1.5, 6.5e-3, 250.0, -7.25e-3, 1e-30]
+    N, K, g = len(scales_f), 64, 64
+    q = np.tile(np.arange(16, dtype=np.uint8), 4)[None, :].repeat(N, 0)
+    packed = O.pack(q)
+    scales = np.array([[O.bf16_rne(s)] for s in scales_f], np.uint16)
+    want = O.dequant(packed, scales, N, K, g)
+    _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
+    got = W.dequant(wd, sd, g).cpu().view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(got, want)
+
+
+# ---------------------------------------------------------------- quantise
+
+def test_quantize_bit_exact_tiny_and_adversarial():
+    W = _W()
+    N, K, g = 1024, 512, 128
+    w = S.make_w_master(N, K, 0, "cpu").numpy()
+    # adversarial groups: all zero, exact ties, +-amax, tiny values
+    w[0, :128] = 0.0
+    w[1, :5] = [7.0, 2.5, -2.5, 3.5, -0.5]
+    w[1, 5:128] = 0.0
+    w[2, :128] = np.linspace(-1, 1, 128, dtype=np.float32)
+    w[3, :128] = 1e-30
+    want_p, want_s = O.quantize(w, g)
+    got_p, got_s = W.quantize(torch.from_numpy(w).cuda(), g)
+    assert np.array_equal(got_p.cpu().numpy(), want_p)
+    assert np.array_equal(got_s.cpu().view(torch.int16).numpy().view(np.uint16), want_s)
+
+
+# ---------------------------------------------------------------- linear
+
+def _run_linear(M, N, K, g, seed=0):
+    W = _W()
+    x, xb, packed, scales = host_case(M, N, K, g, seed, seed + 1)
+    xd, wd, sd = to_device(x, packed, scales)
+    out = W.linear(xd, wd, sd, g)
+    torch.cuda.synchronize()
+    ref = O.linear_rows(xb, packed, scales, N, K, g, nthreads=O.max_threads())
+    return bf16_to_f64(out), ref
+
+
+def test_linear_tiny_config_full():
+    gpu, ref = _run_linear(64, 1024, 512, 128, seed=0)
+    assert_close(gpu, ref, "tiny 64x512x1024")
+
+
+@pytest.mark.parametrize("M,N,K,g", [
+    (1, 128, 128, 128), (5, 200, 256, 128), (32, 384, 512, 128), (33, 300, 384, 128),
+    (257, 130, 640, 128), (300, 1000, 1024, 128), (512, 256, 2048, 128),
+    (40, 256, 256, 64), (100, 512, 1024, 256), (7, 129, 192, 64), (600, 2, 128, 128),
+    (256, 1, 256, 128), (31, 77, 320, 64),
+])
+def test_linear_ragged_shapes(M, N, K, g):
+    gpu, ref = _run_linear(M, N, K, g, seed=M * 7 + N)
+    assert_close(gpu, ref, f"{M}x{K}x{N} g{g}")
+
+
+def test_linear_m_sweep_around_dispatch_threshold():
+    W = _W()
+    N, K, g = 256, 512, 128
+    x, xb, packed, scales = host_case(40, N, K, g, 77, 78)
+    xd, wd, sd = to_device(x, packed, scales)
+    ref = O.linear_rows(xb, packed, scales, N, K, g, nthreads=O.max_threads())
+    for M in range(1, 41):
+        out = W.linear(xd[:M].contiguous(), wd, sd, g)
+        assert_close(bf16_to_f64(out), ref[:M], f"M={M}")
+
+
+def test_linear_guard_bands_untouched():
+    W = _W()
+    M, N, K, g = 67, 258, 256, 128
+    x, xb, packed, scales = host_case(M, N, K, g, 5, 6)
+    xd, wd, sd = to_device(x, packed, scales)
+    guard = 4096
+    buf = torch.full((guard + M * N + guard,), -12345.0, dtype=torch.bfloat16, device="cuda")
+    out = buf[guard:guard + M * N].view(M, N)
+    W.linear(xd, wd, sd, g, out=out)
+    torch.cuda.synchronize()
+    assert (buf[:guard] == -12345.0).all() and (buf[guard + M * N:] == -12345.0).all()
+    ref = O.linear_rows(xb, packed, scales, N, K, g, nthreads=O.max_threads())
+    assert_close(bf16_to_f64(out), ref, "guarded")
+
+
+def test_linear_deterministic():
+    W = _W()
+    x, xb, packed, scales = host_case(300, 512, 1024, 128, 9, 10)
+    xd, wd, sd = to_device(x, packed, scales)
+    a = W.linear(xd, wd, sd)
+    b = W.linear(xd, wd, sd)
+    assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
+def test_linear_stack_chained_and_fresh():
+    W = _W()
+    g, M = 128, 96
+    dims = [(256, 512), (512, 384), (384, 256)]   # (K, N) per layer; layer i+1 reads layer i's out
+    xs, refs, layers = [], [], []
+    x0, x0b, _, _ = host_case(M, 1, dims[0][0], g, 0, 500)
+    xin = x0.cuda()
+    for i, (K, N) in enumerate(dims):
+        w = S.make_w_master(N, K, 600 + i, "cpu").numpy()
+        packed, scales = O.quantize(w, g)
+        _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
+        out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        layers.append((xin, wd, sd, out))
+        refs.append((packed, scales, N, K))
+        xin = out
+    W.linear_stack(layers, M, g)
+    torch.cuda.synchronize()
+    # each layer checked against the oracle on the input that layer actually read
+    for i, (xi, _, _, out) in enumerate(layers):
+        packed, scales, N, K = refs[i]
+        xb = S.bf16_bits(xi)
+        ref = O.linear_rows(xb, packed, scales, N, K, g, nthreads=O.max_threads())
+        assert_close(bf16_to_f64(out), ref, f"stack layer {i}")
+
+
+def test_error_codes_launch_nothing():
+    W = _W()
+    L = W.lib()
+    x = torch.zeros((4, 256), dtype=torch.bfloat16, device="cuda")
+    w = torch.zeros((8, 128), dtype=torch.uint8, device="cuda")
+    s = torch.zeros((8, 2), dtype=torch.bfloat16, device="cuda")
+    o = torch.full((4, 8), 7.0, dtype=torch.bfloat16, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    args = [x.data_ptr(), w.data_ptr(), s.data_ptr(), o.data_ptr()]
+    assert L.w4a16_linear(*args, 0, 8, 256, 128, st) == W.ERR_INVALID_ARG
+    assert L.w4a16_linear(*args, 4, 8, 256, 96, st) == W.ERR_INVALID_ARG       # K % g
+    assert L.w4a16_linear(*args, 4, 8, 256, 32, st) == W.ERR_UNSUPPORTED      # g % 64
+    assert L.w4a16_linear(x.data_ptr() + 2, *args[1:], 4, 8, 256, 128, st) == W.ERR_ALIGNMENT
+    assert L.w4a16_linear(*args[:3], x.data_ptr(), 4, 8, 256, 128, st) == W.ERR_INVALID_ARG  # overlap
+    torch.cuda.synchronize()
+    assert (o == 7.0).all()
