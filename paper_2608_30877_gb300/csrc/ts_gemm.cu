@@ -12,14 +12,15 @@
 // bf16 weight tile never touches shared memory, which keeps shared-memory
 // bandwidth for the x tiles the MMA reads.
 //
-// Warp roles (320 threads):
+// Warp roles (32 * (6 + 4*DQ) threads):
 //   warp 0      TMA producer: x tile [T x 64] and packed weight tile [128 x 32 B]
 //               per stage into a ring of S_SMEM shared-memory stages;
 //   warp 1      allocates tensor memory, one thread issues the MMAs;
-//   warps 2..5  dequantisers: thread = one weight row (its TMEM lane),
-//               32 packed bytes -> 64 bf16 -> 32 TMEM columns per stage,
-//               into a ring of S_TMEM tensor-memory A stages;
-//   warps 6..9  epilogue: tcgen05.ld of the accumulator, fp32 -> bf16,
+//   next 4*DQ   dequantisers, DQ groups of four warps taking stages in turn:
+//               thread = one weight row (its TMEM lane), 32 packed bytes ->
+//               64 bf16 -> 32 TMEM columns per stage, into a ring of S_TMEM
+//               tensor-memory A stages;
+//   last 4      epilogue: tcgen05.ld of the accumulator, fp32 -> bf16,
 //               stores to out.
 // A warp may only touch the 32 TMEM lanes of its sub-partition (warp % 4), so
 // each group of four warps covers all 128 lanes.
@@ -35,7 +36,6 @@ namespace w4a16 {
 
 namespace {
 
-constexpr int kThreads = 320;
 constexpr int kRows = 128;  // weight rows per tile (MMA M)
 constexpr int kBK = 64;     // k per stage (one 128-byte swizzle row of bf16)
 
@@ -81,8 +81,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return r;
 }
 
-template <int T, int S_SMEM, int S_TMEM, int MIN_BLOCKS>
-__global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
+template <int DQ>
+constexpr int threads_for() {
+    return 32 * (6 + 4 * DQ);
+}
+
+template <int T, int S_SMEM, int S_TMEM, int DQ, int MIN_BLOCKS>
+__global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
     w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
     using L = Layout<T, S_SMEM, S_TMEM>;
@@ -111,7 +116,7 @@ __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
             mbar_init(empty_smem(s), 1);
         }
         for (int s = 0; s < S_TMEM; ++s) {
-            mbar_init(full_a(s), 4);  // one arrival per dequant warp
+            mbar_init(full_a(s), 4);  // one arrival per dequant warp of the stage's group
             mbar_init(empty_a(s), 1);
         }
         mbar_init(d_full, 1);
@@ -208,29 +213,46 @@ __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
                 }
             }
         }
-    } else if (warp < 6) {
+    } else if (warp < 2 + 4 * DQ) {
         // ------------------------------------------------------------ dequantisers
+        const int dgrp = (warp - 2) >> 2;  // which group of four warps
         const int sub = warp & 3;
         const int r = sub * 32 + lane;
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
-        uint32_t it = 0;
-        bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+        // stages per scale group; a shift when that is a power of two
+        const int spg = p.g / kBK;
+        const int spg_shift = (spg & (spg - 1)) == 0 ? __ffs(spg) - 1 : -1;
+        auto grp_of = [&](int kt) { return spg_shift >= 0 ? (kt >> spg_shift) : kt / spg; };
+        // scale row of the tile processed at per-CTA tile index j (nullptr: none)
+        auto scale_row = [&](int j) -> const uint16_t* {
+            const int tile = blockIdx.x + j * gridDim.x;
+            if (tile >= p.num_tiles) return nullptr;
             int tt, wt;
             tile_coords(tile, p, tt, wt);
             const int n = wt * kRows + r;
-            const bool valid = n < p.N;
-            const uint16_t* srow = p.scales + static_cast<int64_t>(valid ? n : 0) * KG;
-            uint16_t s_cur = valid ? __ldg(srow) : 0;
-            uint16_t s_nxt = (valid && KG > 1) ? __ldg(srow + 1) : 0;
-            int cur_grp = 0;
+            return n < p.N ? p.scales + static_cast<int64_t>(n) * KG : nullptr;
+        };
+        // one-stage lookahead: the scale for this warp's next stage is loaded
+        // while the current one is dequantised
+        auto load_scale = [&](uint32_t i) -> uint16_t {
+            const int j = static_cast<int>(i / static_cast<uint32_t>(KT));
+            const int kt = static_cast<int>(i - static_cast<uint32_t>(j) * KT);
+            const uint16_t* row = scale_row(j);
+            return row ? __ldg(row + grp_of(kt)) : static_cast<uint16_t>(0);
+        };
+        uint32_t it = 0;
+        bool ok = true;
+        uint16_t s_next = load_scale(static_cast<uint32_t>(dgrp));
+        for (int j = 0, tile = blockIdx.x; ok && tile < p.num_tiles; ++j, tile += gridDim.x) {
+            const uint16_t* srow = scale_row(j);
             for (int kt = 0; kt < KT; ++kt, ++it) {
-                const int grp = (kt * kBK) / p.g;
-                if (grp != cur_grp) {
-                    s_cur = s_nxt;
-                    cur_grp = grp;
-                    s_nxt = (valid && grp + 1 < KG) ? __ldg(srow + grp + 1) : 0;
-                }
+                if (static_cast<int>(it % DQ) != dgrp) continue;
+                const uint16_t s_cur = s_next;
+                const int kt2 = kt + DQ;
+                if (kt2 < KT)
+                    s_next = srow ? __ldg(srow + grp_of(kt2)) : static_cast<uint16_t>(0);
+                else
+                    s_next = load_scale(it + DQ);
                 const int s = it % S_SMEM;
                 const int sa = it % S_TMEM;
                 if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status) ||
@@ -326,25 +348,28 @@ __global__ void __launch_bounds__(kThreads, MIN_BLOCKS)
     if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
 }
 
-template <int T, int S_SMEM, int S_TMEM, int MIN_BLOCKS>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int MIN_BLOCKS>
 cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
                            int grid, cudaStream_t stream) {
     using L = Layout<T, S_SMEM, S_TMEM>;
-    auto kern = w4a16_ts_kernel<T, S_SMEM, S_TMEM, MIN_BLOCKS>;
+    auto kern = w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, MIN_BLOCKS>;
     // Idempotent; cheap enough to repeat per launch and per device.
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    kern<<<grid, threads_for<DQ>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
     return cudaGetLastError();
 }
 
 // Large M: 256 tokens per tile, 6 stages of (32 KB x + 4 KB packed weights),
 // tensor memory = 256 accumulator columns + 6 x 32 A columns.
-constexpr int kGemmT = 256, kGemmSS = 6, kGemmST = 6;
+#ifndef W4A16_GEMM_DQ
+#define W4A16_GEMM_DQ 2
+#endif
+constexpr int kGemmT = 256, kGemmSS = 6, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
-constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3;
+constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1;
 
 }  // namespace
 
@@ -358,8 +383,8 @@ int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
                       const TsParams& p, int grid, cudaStream_t stream) {
     if (v == TsVariant::kGemm256)
-        return launch_variant<kGemmT, kGemmSS, kGemmST, 1>(tx, tw, p, grid, stream);
-    return launch_variant<kGemvT, kGemvSS, kGemvST, 3>(tx, tw, p, grid, stream);
+        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, 1>(tx, tw, p, grid, stream);
+    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, 3>(tx, tw, p, grid, stream);
 }
 
 }  // namespace w4a16
