@@ -253,7 +253,7 @@ class LinearWorkload:
 
 # ----------------------------------------------------------------- CPU oracle
 
-def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 64):
+def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 2048):
     """Times the oracle on `r` token rows x N_rows weight rows of one K-deep
     linear with seeded inputs; grows r until the sample takes ~target_s.
     Returns (MAC/s, description, threads)."""
@@ -271,11 +271,11 @@ def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 64):
         dt = time.perf_counter() - t0
         spent += dt
         macs_r = r * N_rows * K
-        if dt >= target_s / 3 or r >= rows_max or spent >= target_s:
+        if dt >= target_s / 3 or r >= rows_max or spent >= 2 * target_s:
             desc = (f"oracle fp64 linear, {r} token rows x {N_rows} weight rows x K={K} "
                     f"({macs_r / 1e9:.2f} GMAC) in {dt:.2f} s on {threads} threads")
             return macs_r / dt, desc, threads
-        r = min(rows_max, max(r + 1, int(r * (target_s / 3) / max(dt, 1e-3))))
+        r = min(rows_max, max(r + 1, int(r * (target_s / 2) / max(dt, 1e-3))))
 
 
 def stack_macs_per_pair(tokens=1024, layers=96):

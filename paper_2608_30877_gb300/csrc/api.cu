@@ -34,6 +34,7 @@ std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 8;
+bool g_small_m_streaming = true;
 
 // Per-device set-up, done once with the device current.
 int device_state(DeviceState** out) {
@@ -51,6 +52,9 @@ int device_state(DeviceState** out) {
                 q != cudaDriverEntryPointSuccess || fn == nullptr)
                 return W4A16_ERR_CUDA;
             g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+            if (const char* e = std::getenv("W4A16_SMALL_M_TILED")) {
+                if (e[0] == '1') g_small_m_streaming = false;
+            }
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
                 if (v > 0 && v <= 4096) g_group_t = v;
@@ -119,9 +123,43 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
     return r == CUDA_SUCCESS ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
+// Small M with K a multiple of 128: the streaming kernel (rows spread evenly
+// over the SMs).
+int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
+                int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
+    const int T = gemv_tokens_per_tile(M);
+    const int RB = gemv_rows_per_cta(N, st.sm_count);
+    alignas(64) CUtensorMap tx;
+    alignas(64) CUtensorMap tw;
+    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
+                       CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != W4A16_OK) return rc;
+    rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 64, RB / 2,
+                   CU_TENSOR_MAP_SWIZZLE_64B);
+    if (rc != W4A16_OK) return rc;
+    GemvParams p;
+    p.scales = static_cast<const uint16_t*>(s);
+    p.out = static_cast<uint16_t*>(out);
+    p.status = st.status;
+    p.M = static_cast<int>(M);
+    p.N = static_cast<int>(N);
+    p.K = static_cast<int>(K);
+    p.g = static_cast<int>(g);
+    p.rows_per_cta = RB;
+    p.num_chunks = static_cast<int>((N + RB - 1) / RB);
+    p.nt = (RB + 127) / 128;
+    p.m4 = 1u << 28;
+    p.m8 = 1u << 24;
+    p.m12 = 1u << 20;
+    return gemv_launch(&tx, &tw, p, st.sm_count, stream) == cudaSuccess ? W4A16_OK
+                                                                         : W4A16_ERR_CUDA;
+}
+
 // Validated arguments -> one kernel launch.
 int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                   int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
+    if (M <= 32 && K % 128 == 0 && g_small_m_streaming)
+        return launch_gemv(st, x, w, s, out, M, N, K, g, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
     alignas(64) CUtensorMap tx;

@@ -34,6 +34,26 @@ int ts_grid(TsVariant v, const TsParams& p, int sm_count);
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                       const TsParams& p, int grid, cudaStream_t stream);
 
+// Parameters of the small-M streaming kernel (gemv_rows.cu).
+struct GemvParams {
+    const uint16_t* scales;  // bf16 bits [N, K/g]
+    uint16_t* out;           // bf16 bits [M, N]
+    int* status;
+    int M, N, K, g;
+    int rows_per_cta;        // RB: weight rows per CTA chunk, multiple of 16, <= 384
+    int num_chunks;          // ceil(N / RB)
+    int nt;                  // MMA tiles per chunk: ceil(RB / 128)
+    // 2^28, 2^24, 2^20: multipliers that turn mul.hi into shifts by 4, 8, 12
+    // (run-time values so that the shifts stay on the FMA pipe)
+    uint32_t m4, m8, m12;
+};
+
+// RB for N rows spread over the SMs; tokens per tile for M.
+int gemv_rows_per_cta(int64_t N, int sm_count);
+int gemv_tokens_per_tile(int64_t M);
+cudaError_t gemv_launch(const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
+                        const GemvParams& p, int sm_count, cudaStream_t stream);
+
 cudaError_t launch_dequant(const uint8_t* w, const uint16_t* scales, uint16_t* wd, int64_t N,
                            int64_t K, int64_t g, cudaStream_t stream);
 cudaError_t launch_quantize(const float* w, uint8_t* packed, uint16_t* scales, int64_t N,

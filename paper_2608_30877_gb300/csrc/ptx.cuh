@@ -115,6 +115,34 @@ __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatil
     }
 }
 
+// Warp-wide wait for long, latency-tolerant waits (an epilogue waiting for a
+// whole tile's MMAs): between polls the warp sleeps sleep_ns, so it takes no
+// issue slots from the warps doing the work.
+__device__ __forceinline__ bool wait_warp_sleep(uint32_t bar, uint32_t parity,
+                                                volatile int* abort_flag, int* status,
+                                                uint32_t sleep_ns) {
+    const uint32_t lane = threadIdx.x & 31u;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0;; ++it) {
+        const bool done = mbar_try_wait(bar, parity);
+        if (__all_sync(0xffffffffu, done)) return true;
+        __nanosleep(sleep_ns);
+        if ((it & 7u) == 7u) {
+            int give_up = 0;
+            if (lane == 0) {
+                if (*abort_flag) {
+                    give_up = 1;
+                } else if (it > kWaitIterCap || global_timer_ns() - t0 > kWaitLimitNs) {
+                    *abort_flag = 1;
+                    atomicExch(status, 5 /* W4A16_ERR_TIMEOUT */);
+                    give_up = 1;
+                }
+            }
+            if (__shfl_sync(0xffffffffu, give_up, 0)) return false;
+        }
+    }
+}
+
 // ---------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {

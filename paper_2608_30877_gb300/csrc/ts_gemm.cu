@@ -37,6 +37,10 @@ namespace w4a16 {
 namespace {
 
 constexpr int kRows = 128;  // weight rows per tile (MMA M)
+#ifndef W4A16_EPI_SLEEP_NS
+#define W4A16_EPI_SLEEP_NS 256
+#endif
+constexpr uint32_t kEpilogueSleepNs = W4A16_EPI_SLEEP_NS;
 constexpr int kBK = 64;     // k per stage (one 128-byte swizzle row of bf16)
 
 template <int T, int S_SMEM, int S_TMEM>
@@ -291,7 +295,8 @@ __global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
         for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++tcount) {
             int tt, wt;
             tile_coords(tile, p, tt, wt);
-            if (!wait_warp(d_full, tcount & 1u, abort_flag, p.status)) break;
+            if (!wait_warp_sleep(d_full, tcount & 1u, abort_flag, p.status, kEpilogueSleepNs))
+                break;
             tc_fence_after();
             const int n = wt * kRows + sub * 32 + lane;
 #pragma unroll 1
@@ -366,7 +371,10 @@ cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const T
 #ifndef W4A16_GEMM_DQ
 #define W4A16_GEMM_DQ 2
 #endif
-constexpr int kGemmT = 256, kGemmSS = 6, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ;
+#ifndef W4A16_GEMM_SS
+#define W4A16_GEMM_SS 6
+#endif
+constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
 constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1;

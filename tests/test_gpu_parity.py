@@ -178,3 +178,14 @@ def test_error_codes_launch_nothing():
     assert L.w4a16_linear(*args[:3], x.data_ptr(), 4, 8, 256, 128, st) == W.ERR_INVALID_ARG  # overlap
     torch.cuda.synchronize()
     assert (o == 7.0).all()
+
+
+@pytest.mark.parametrize("M,N,K,g", [
+    (1, 1, 128, 128), (3, 100, 256, 128), (8, 1000, 1024, 128), (16, 4096, 512, 128),
+    (17, 1234, 384, 128), (32, 8192, 256, 64), (32, 50000, 128, 128), (9, 77, 2048, 256),
+])
+def test_small_m_streaming_kernel_shapes(M, N, K, g):
+    """M <= 32 with K a multiple of 128 runs the row-range streaming kernel:
+    ragged row ranges, 1-3 MMA tiles per CTA, 16 and 32 token columns."""
+    gpu, ref = _run_linear(M, N, K, g, seed=3 * M + N)
+    assert_close(gpu, ref, f"{M}x{K}x{N} g{g}")
