@@ -123,8 +123,8 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
     return r == CUDA_SUCCESS ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
-// Small M with K a multiple of 128: the streaming kernel (rows spread evenly
-// over the SMs).
+// M <= 16 with g = 128: the streaming kernel (rows spread evenly over the
+// SMs).
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                 int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
     const int T = gemv_tokens_per_tile(M);
@@ -158,7 +158,7 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
 // Validated arguments -> one kernel launch.
 int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                   int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
-    if (M <= 32 && K % 128 == 0 && g_small_m_streaming)
+    if (M <= 16 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
