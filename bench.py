@@ -33,19 +33,40 @@ if ROOT not in sys.path:
 
 METRIC = "W4A16 GEMM TFLOP/s & % of roofline; scored pairs/s on 175B-class linear stack"
 
-# ncu DRAM traffic (read + write bytes per launch) of the fused kernel, keyed by
-# the hash of the kernel sources the counters were taken on (see profiles/).
-# A mismatch (the kernel changed since) reports traffic as null.
-NCU_TRAFFIC = {}
+# ncu DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum per launch) of
+# the timed kernel, from the captures summarised in profiles/, keyed by the
+# workload and by a hash of the kernel's sources at capture time: once the
+# kernel changes the hash no longer matches and traffic is reported as null.
+NCU_TRAFFIC = {
+    # 384 launches of the timed stack step (launch list with DRAM counters)
+    ("stack", "ts", "e4bf59b3aed036fa"): 37.028e9,
+    # QKV prefill 4096x12288x36864, one launch (full capture)
+    ("qkv", "ts", "e4bf59b3aed036fa"): 1.174e9 + 0.294e9,
+    # small-M readout, M = 8, 12288x49152 (full capture)
+    ("gemv", "gemv", "98e5e3730890bf2f"): 0.3237e9 + 0.0034e9,
+}
+
+KERNEL_FILES = {"ts": ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"),
+                "gemv": ("gemv_rows.cu", "dequant.cuh", "ptx.cuh")}
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(kind: str = "ts") -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_30877_gb300", "csrc")
-    for name in ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"):
+    for name in KERNEL_FILES[kind]:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
+
+
+def ncu_traffic(config: str, m: int):
+    if config == "gemv":
+        if m > 8:  # the capture is of the M <= 8 instantiation
+            return None
+        kind = "gemv"
+    else:
+        kind = "ts"
+    return NCU_TRAFFIC.get((config, kind, kernel_source_hash(kind)))
 
 
 def load_peaks() -> dict:
@@ -419,7 +440,7 @@ def main():
         achieved = wl.flops / step_s / 1e12
         peak = peaks["bf16_tflops_sustained"] if args.config == "stack" else peaks["bf16_tflops"]
         roof = {"bound": "tensor", "unit": "TFLOP/s"}
-    traffic = NCU_TRAFFIC.get((args.config, kernel_source_hash()))
+    traffic = ncu_traffic(args.config, args.m)
     roof.update({"achieved": achieved, "peak": peak, "frac": achieved / peak,
                  "traffic": traffic, "peak_source": peaks["source"] + (
                      " bf16_tflops_sustained" if args.config == "stack" else

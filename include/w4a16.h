@@ -69,8 +69,10 @@ typedef enum {
  *   w_packed_u8  [N, K/2] uint8, device, layout above
  *   scales_bf16  [N, K/g] bf16, device
  *   out_bf16     [M, N]   bf16, device, written in full
- * M <= 32 runs the bandwidth-bound small-M kernel, larger M the tensor-core
- * GEMM; both are the same fused dequant + tcgen05 MMA design.
+ * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 16 with
+ * g = 128 runs the bandwidth-bound row-range streaming kernel; other small
+ * M run the tcgen05 kernel with 32-token tiles.  All produce the same
+ * result up to fp32 summation order.
  */
 int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
                  void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,
@@ -121,6 +123,17 @@ int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales_bf16,
  * W4A16_ERR_TIMEOUT or W4A16_ERR_CUDA.
  */
 int w4a16_get_device_error(void* stream);
+
+/*
+ * Test hook for the kernels' bounded waits; the paper has no counterpart.
+ * Launches one CTA on `stream` that waits on a shared-memory mbarrier nothing
+ * arrives on, giving up after limit_ns nanoseconds of global time
+ * (1e3 <= limit_ns <= 1e9, else W4A16_ERR_INVALID_ARG).  On giving up it
+ * records W4A16_ERR_TIMEOUT in the device status word and returns -- the same
+ * path the production kernels take -- so that w4a16_get_device_error reports
+ * it and the context stays usable.
+ */
+int w4a16_selftest_wait_timeout(int64_t limit_ns, void* stream);
 
 /* Static text for a status code; never NULL. */
 const char* w4a16_status_string(int status);

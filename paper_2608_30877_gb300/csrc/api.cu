@@ -1,6 +1,7 @@
 // C ABI of the library (declared in include/w4a16.h): argument validation,
 // TMA descriptor encoding, kernel dispatch and the device status word.
 #include "internal.h"
+#include "ptx.cuh"
 #include "w4a16.h"
 
 #include <cuda.h>
@@ -16,6 +17,26 @@ namespace {
 // Set by kernels when a bounded wait runs out; read and cleared by
 // w4a16_get_device_error.
 __device__ int g_status_word;
+
+// One thread waits on an mbarrier that nothing arrives on, until limit_ns of
+// global time have passed, then records a timeout like the real kernels.
+__global__ void selftest_wait_kernel(uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(smem_u32(&bar), 0)) {
+            if (global_timer_ns() - t0 > limit_ns) {
+                atomicExch(&g_status_word, W4A16_ERR_TIMEOUT);
+                break;
+            }
+        }
+    }
+}
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -275,6 +296,16 @@ extern "C" int w4a16_get_device_error(void* stream) {
         cudaMemcpy(st->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
         return W4A16_ERR_CUDA;
     return v == 0 ? W4A16_OK : v;
+}
+
+extern "C" int w4a16_selftest_wait_timeout(int64_t limit_ns, void* stream) {
+    if (limit_ns < 1000 || limit_ns > 1000000000) return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    const int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<uint64_t>(limit_ns));
+    return cudaGetLastError() == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
 extern "C" const char* w4a16_status_string(int status) {

@@ -53,11 +53,12 @@ def lib() -> ctypes.CDLL:
         L.w4a16_dequant.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_quantize.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_get_device_error.argtypes = [p]
+        L.w4a16_selftest_wait_timeout.argtypes = [i64, p]
         L.w4a16_status_string.argtypes = [ctypes.c_int]
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
         for f in ("w4a16_linear", "w4a16_linear_stack", "w4a16_dequant", "w4a16_quantize",
-                  "w4a16_get_device_error"):
+                  "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -155,6 +156,12 @@ def quantize(w: torch.Tensor, g: int = 128, stream=None):
     _check("w4a16_quantize", lib().w4a16_quantize(w.data_ptr(), packed.data_ptr(),
                                                   scales.data_ptr(), N, K, g, _stream(stream)))
     return packed, scales
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
+    """Launch the bounded-wait self test (see include/w4a16.h)."""
+    _check("w4a16_selftest_wait_timeout",
+           lib().w4a16_selftest_wait_timeout(int(limit_ns), _stream(stream)))
 
 
 def get_device_error(stream=None) -> int:

@@ -1,0 +1,77 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case compiles a copy of oracle/w4a16_oracle.c with one planted mistake
+(swapped nibbles, dropped zero point, wrong group index, round-half-away,
+truncating bf16 rounding, fp32 accumulation, wrong activation row), points
+the oracle module at it and runs the pins: at least one must fail.  The
+mistakes live only in temporary copies on the CPU."""
+import ctypes
+import os
+import subprocess
+import tempfile
+
+import pytest
+
+from oracle import oracle as O
+from tests import test_oracle_pins as P
+
+SRC = os.path.join(os.path.dirname(O.__file__), "w4a16_oracle.c")
+
+MUTANTS = {
+    "swapped_nibbles": [("(k % 2 == 0) ? (b & 0x0F) : (b >> 4)", "(k % 2 == 0) ? (b >> 4) : (b & 0x0F)")],
+    "no_zero_point": [("(float)(q - 8) * s", "(float)(q) * s")],
+    "group_index_mod": [("scales[n * KG + k / g]", "scales[n * KG + (k % KG)]")],
+    "round_half_away": [("nearbyintf(grp[t] / s)", "roundf(grp[t] / s)")],
+    "bf16_truncates": [("u += 0x7FFFu + kept_lsb;", "u += 0u * kept_lsb;")],
+    "fp32_accumulate": [("double acc = 0.0;", "float acc = 0.0f;")],
+    "wrong_x_row": [("const uint16_t* xrow = x + rows[r] * K;", "const uint16_t* xrow = x;")],
+}
+
+PINS = [
+    P.test_bf16_rne_hand_values,
+    P.test_unpack_every_byte,
+    P.test_dequant_table_all_codes_against_exact_product,
+    P.test_dequant_rounding_cases_by_hand,
+    P.test_dequant_group_index,
+    P.test_linear_hand_computed_2x3x256,
+    P.test_linear_power_of_two_scales_equals_textbook_matmul,
+    P.test_linear_invariants,
+    P.test_linear_brute_force_small,
+    P.test_quantize_hand_example,
+    P.test_quantize_rounds_half_to_even_and_zero_group,
+    P.test_quantize_error_bound_and_code_range,
+]
+
+
+def _build_mutant(name, edits, outdir):
+    src = open(SRC).read()
+    for old, new in edits:
+        assert old in src, (name, old)
+        src = src.replace(old, new)
+    c = os.path.join(outdir, f"{name}.c")
+    so = os.path.join(outdir, f"{name}.so")
+    open(c, "w").write(src)
+    subprocess.run(["gcc", "-O2", "-fPIC", "-shared", "-fopenmp", "-fno-fast-math",
+                    "-ffp-contract=off", "-o", so, c, "-lm"], check=True)
+    return so
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(name, monkeypatch):
+    good = O.lib()
+    with tempfile.TemporaryDirectory() as d:
+        so = _build_mutant(name, MUTANTS[name], d)
+        mut = ctypes.CDLL(so)
+        for fn in ("oracle_bf16_rne", "oracle_bf16_to_f32", "oracle_unpack", "oracle_pack",
+                   "oracle_quantize", "oracle_dequant", "oracle_linear_rows",
+                   "oracle_linear_points", "oracle_max_threads"):
+            getattr(mut, fn).argtypes = getattr(good, fn).argtypes
+            getattr(mut, fn).restype = getattr(good, fn).restype
+        monkeypatch.setattr(O, "_lib", mut)
+        failed = []
+        for pin in PINS:
+            try:
+                pin()
+            except AssertionError:
+                failed.append(pin.__name__)
+        assert failed, f"no pin caught the planted mistake {name}"
