@@ -69,10 +69,10 @@ typedef enum {
  *   w_packed_u8  [N, K/2] uint8, device, layout above
  *   scales_bf16  [N, K/g] bf16, device
  *   out_bf16     [M, N]   bf16, device, written in full
- * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 16 with
+ * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 32 with
  * g = 128 runs the bandwidth-bound row-range streaming kernel; other small
- * M run the tcgen05 kernel with 32-token tiles.  All produce the same
- * result up to fp32 summation order.
+ * M (g != 128) run the tcgen05 kernel with 32-token tiles.  All produce the
+ * same result up to fp32 summation order.
  */
 int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
                  void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,

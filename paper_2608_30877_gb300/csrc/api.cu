@@ -144,7 +144,7 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
     return r == CUDA_SUCCESS ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
-// M <= 16 with g = 128: the streaming kernel (rows spread evenly over the
+// M <= 32 with g = 128: the streaming kernel (rows spread evenly over the
 // SMs).
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                 int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
@@ -169,9 +169,6 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
     p.rows_per_cta = RB;
     p.num_chunks = static_cast<int>((N + RB - 1) / RB);
     p.nt = (RB + 127) / 128;
-    p.m4 = 1u << 28;
-    p.m8 = 1u << 24;
-    p.m12 = 1u << 20;
     return gemv_launch(&tx, &tw, p, st.sm_count, stream) == cudaSuccess ? W4A16_OK
                                                                          : W4A16_ERR_CUDA;
 }
@@ -179,7 +176,7 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
 // Validated arguments -> one kernel launch.
 int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                   int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
-    if (M <= 16 && g == 128 && K % 128 == 0 && g_small_m_streaming)
+    if (M <= 32 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);

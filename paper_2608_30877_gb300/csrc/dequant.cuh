@@ -49,32 +49,9 @@ __device__ __forceinline__ void dequant_word(uint32_t w, uint32_t s2, uint32_t* 
     }
 }
 
-__device__ __forceinline__ uint32_t mulhi_u32(uint32_t a, uint32_t b) {
-    uint32_t r;
-    asm("mul.hi.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
-    return r;
-}
-
-// Same values as dequant_word, in the pair order (k = j, k = j + 4):
-// out[j] = (wd(k=j) low half, wd(k=j+4) high half), j = 0..3.  Each pair is
-// one mask of a shifted copy of the word (nibbles j and j+4 sit 16 bits
-// apart), so the integer pipe does one LOP3 per pair; the shifts by 4, 8 and
-// 12 are multiply-high by m4 = 2^28, m8 = 2^24, m12 = 2^20, which the caller
-// passes in as run-time values so that they execute on the FMA pipe.  A
-// consumer of these pairs must present the other operand in the same order.
-__device__ __forceinline__ void dequant_word_interleaved(uint32_t w, uint32_t s2, uint32_t m4,
-                                                         uint32_t m8, uint32_t m12,
-                                                         uint32_t* out) {
-    const uint32_t src[4] = {w, mulhi_u32(w, m4), mulhi_u32(w, m8), mulhi_u32(w, m12)};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const uint32_t t = (src[j] & 0x000F000Fu) | 0x43004300u;  // (128 + q_j, 128 + q_j+4)
-        out[j] = bf16x2_mul(bf16x2_sub(t, 0x43084308u), s2);
-    }
-}
-
 // Puts the 8 bf16 of a 16-byte chunk (x0..x7) in the pair order
-// (x0,x4),(x1,x5),(x2,x6),(x3,x7) used by dequant_word_interleaved.
+// (x0,x4),(x1,x5),(x2,x6),(x3,x7): the order in which one packed word yields
+// its codes when each pair is masked out of a shifted copy of the word.
 __device__ __forceinline__ uint4 interleave_chunk(uint4 c) {
     uint4 r;
     r.x = prmt_b32(c.x, c.z, 0x5410u);

@@ -1,4 +1,4 @@
-// Small-M (M <= 16) int4-dequant + matmul for sm_103a: the bandwidth-bound
+// Small-M (M <= 32) int4-dequant + matmul for sm_103a: the bandwidth-bound
 // regime where the whole packed weight matrix streams from HBM once per call.
 //
 // Design, GB300-first:
@@ -7,25 +7,26 @@
 //     same number of bytes -- no tile-count quantisation;
 //   - one shared-memory stage covers 128 k = one scale group (g = 128): two
 //     TMA boxes of RB/2 rows x 64 B of packed weights (64-byte swizzle) and
-//     two 128-byte-swizzled boxes of x (T = 8 or 16 token rows; rows >= M
+//     two 128-byte-swizzled boxes of x (T = 8, 16 or 32 token rows; rows >= M
 //     are TMA zero fill); warp 0 keeps S stages in flight;
+//   - warp 1 reorders each staged x chunk once, in place, into the pair order
+//     the weight codes come out in (below), for all compute warps;
 //   - one compute warp per 32 weight rows (two m16 tiles).  Its threads
 //     unpack codes straight into the A fragments of mma.sync.m16n8k16 (bf16
 //     in, fp32 out): nothing is staged in shared or tensor memory and there
-//     is no hand-off between warps inside the K loop.  With 8-16 token
+//     is no hand-off between warps inside the K loop.  With 8-32 token
 //     columns an MMA carries little work, and the fine-grained tcgen05
 //     hand-offs (TMEM stores, commits, barrier round trips) would cost more
 //     than the math;
-//   - each 8-code word is unpacked as the pairs (k, k+4) into the exact bf16
-//     128 + q: one integer-pipe op per pair, the shifts as multiply-high on
-//     the FMA pipe, no per-weight arithmetic.  The thread puts its x chunks
-//     in the same pair order in registers.  Per group the MMA sums
-//     d = sum x * (128 + q); one more MMA per k step with the constant A =
-//     -136 (exact in bf16) sums db = -136 * sum x, already in the layout of
-//     d, and acc += s * (d + db) applies zero point and scale in fp32;
-//   - reading an MMA accumulator waits for every MMA the warp still has in
-//     flight, so G consecutive groups accumulate into G separate register
-//     sets and are folded together: one drain per G groups;
+//   - each 8-code word is unpacked as the pairs (k, k+4): a mask of the word
+//     shifted by 4j gives the exact bf16 pair 128 + q, one bf16x2 subtraction
+//     of 136 the exact q - 8 -- two integer-pipe instructions and one
+//     half-precision one per pair.  Per group the MMA sums d = sum x (q - 8)
+//     in fp32 and acc += s * d applies the scale;
+//   - the K loop is unrolled over the S stage slots, so every shared-memory
+//     address is a per-thread base plus an immediate; a chunk's stage count is
+//     padded to a multiple of S with empty stages that only cycle the
+//     barriers;
 //   - each CTA walks K from its own starting group, so the CTAs do not all
 //     read the same x slice from L2 at the same moment.
 // Fragment k mapping: within a 128-k stage, thread quad index c owns k in
@@ -39,14 +40,24 @@
 
 #include <cuda_bf16.h>
 
-#ifndef W4A16_GEMV_G1
-#define W4A16_GEMV_G1 1
+// Stage slots and unroll (scale block) per token-tile count.
+#ifndef W4A16_GEMV_S1
+#define W4A16_GEMV_S1 8
 #endif
-#ifndef W4A16_GEMV_G2
-#define W4A16_GEMV_G2 1
+#ifndef W4A16_GEMV_U1
+#define W4A16_GEMV_U1 4
 #endif
-#ifndef W4A16_GEMV_TPW
-#define W4A16_GEMV_TPW 2
+#ifndef W4A16_GEMV_S2
+#define W4A16_GEMV_S2 8
+#endif
+#ifndef W4A16_GEMV_U2
+#define W4A16_GEMV_U2 4
+#endif
+#ifndef W4A16_GEMV_S4
+#define W4A16_GEMV_S4 4
+#endif
+#ifndef W4A16_GEMV_U4
+#define W4A16_GEMV_U4 4
 #endif
 
 namespace w4a16 {
@@ -55,9 +66,13 @@ namespace {
 
 constexpr int kRowsMax = 352;  // 11 compute warps of 32 rows
 constexpr int kBKS = 128;      // k per shared-memory stage = one scale group
+constexpr int kRowsPerWarp = 32;
+constexpr int kFirstComputeWarp = 2;
+constexpr int kMaxThreads = 32 * (kFirstComputeWarp + kRowsMax / kRowsPerWarp);
 
 template <int NT, int S>
 struct GLayout {
+    static_assert(S >= 2, "stage slots");
     static constexpr int T = 8 * NT;                            // token rows staged
     static constexpr int X_BOX = T * 128;                       // one 64-k box of x
     static constexpr int X_BYTES = 2 * X_BOX;
@@ -66,13 +81,15 @@ struct GLayout {
     static constexpr int X_OFF = 0;
     static constexpr int W_OFF = S * X_BYTES;
     static constexpr int BAR_OFF = W_OFF + S * W_BYTES;
-    static constexpr int NBARS = 2 * S;  // full_tma, empty_smem
+    static constexpr int NBARS = 3 * S;  // full (TMA), ready (x reordered), empty
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;
     static_assert(X_BOX % 1024 == 0, "x boxes keep the 128-byte swizzle phase");
     static_assert(W_HALF % 1024 == 0, "weight boxes keep the 64-byte swizzle phase");
+    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
 };
 
+// d += A * B: m16n8k16, bf16 inputs, fp32 accumulators.
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
                                                uint32_t a2, uint32_t a3, uint32_t b0,
                                                uint32_t b1) {
@@ -83,24 +100,85 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Biased codes (128 + q) as exact bf16 pairs (k = j, k = j + 4) of one packed
-// word (the shifts are multiply-high by run-time 2^28, 2^24, 2^20).
-__device__ __forceinline__ void codes_biased(uint32_t w, uint32_t m4, uint32_t m8, uint32_t m12,
-                                             uint32_t* out) {
-    out[0] = (w & 0x000F000Fu) | 0x43004300u;
-    out[1] = (mulhi_u32(w, m4) & 0x000F000Fu) | 0x43004300u;
-    out[2] = (mulhi_u32(w, m8) & 0x000F000Fu) | 0x43004300u;
-    out[3] = (mulhi_u32(w, m12) & 0x000F000Fu) | 0x43004300u;
+// d = A * B: a zero C operand starts a fresh accumulator without clearing it.
+__device__ __forceinline__ void mma_bf16_16816_first(float (&d)[4], uint32_t a0, uint32_t a1,
+                                                     uint32_t a2, uint32_t a3, uint32_t b0,
+                                                     uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
+        : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
 }
 
-__device__ __forceinline__ float bf16_bits_to_float(uint32_t h) {
-    return __uint_as_float(h << 16);
+// (w >> n) & 0x000F000F | 0x43004300 as one shift and one three-input logic
+// op; written out so that the mask and the bias merge into a single LOP3.
+template <int n>
+__device__ __forceinline__ uint32_t nibble_pair_biased(uint32_t w) {
+    uint32_t r;
+    if constexpr (n == 0) {
+        asm("lop3.b32 %0, %1, 0x000F000F, 0x43004300, 0xEA;" : "=r"(r) : "r"(w));
+    } else {
+        asm("{\n\t.reg .b32 t;\n\t"
+            "shr.b32 t, %1, %2;\n\t"
+            "lop3.b32 %0, t, 0x000F000F, 0x43004300, 0xEA;\n\t}"
+            : "=r"(r)
+            : "r"(w), "n"(n));
+    }
+    return r;
 }
 
-// 12 warps at most with two tiles per warp (384 threads, up to 144
-// registers), 23 with one (736 threads, up to 80).
-template <int NT, int S, int G, int TPW>
-__global__ void __launch_bounds__(TPW == 2 ? 384 : 736, 1)
+// Codes minus the zero point, q - 8, as exact bf16 pairs (k = j, k = j + 4)
+// of one packed word: nibbles j and j + 4 sit 16 bits apart, so the mask of
+// the word shifted by 4j gives (128 + q_j, 128 + q_j+4), and subtracting 136
+// (all exact in bf16) the signed codes.
+__device__ __forceinline__ void codes_signed(uint32_t w, uint32_t* out) {
+    out[0] = bf16x2_sub(nibble_pair_biased<0>(w), 0x43084308u);
+    out[1] = bf16x2_sub(nibble_pair_biased<4>(w), 0x43084308u);
+    out[2] = bf16x2_sub(nibble_pair_biased<8>(w), 0x43084308u);
+    out[3] = bf16x2_sub(nibble_pair_biased<12>(w), 0x43084308u);
+}
+
+// Scale e of a block held as bf16 pairs, as fp32: a low half by an integer
+// multiply by 2^16 (FMA pipe), a high half by a mask.
+// (e is a constant once the stage loop is unrolled.)
+template <int W>
+__device__ __forceinline__ float scale_at(const uint32_t (&blk)[W], int e) {
+    const uint32_t w = blk[e >> 1];
+    if ((e & 1) == 0) {
+        uint32_t r;
+        asm("mul.lo.u32 %0, %1, 65536;" : "=r"(r) : "r"(w));
+        return __uint_as_float(r);
+    } else {
+        return __uint_as_float(w & 0xFFFF0000u);
+    }
+}
+
+// Shared-memory loads by 32-bit address (volatile: they stay after the
+// barrier waits that guard them).
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// NT: 8-token MMA column tiles (T = 8 NT staged token rows); S: stage slots;
+// U: stages per unrolled round of the K loop, and scale groups per load (a
+// divisor of S).
+template <int NT, int S, int U>
+__global__ void __launch_bounds__(kMaxThreads, 1)
     w4a16_gemv_kernel(const __grid_constant__ CUtensorMap tmap_x,
                       const __grid_constant__ CUtensorMap tmap_w, const GemvParams p) {
     using L = GLayout<NT, S>;
@@ -112,19 +190,19 @@ __global__ void __launch_bounds__(TPW == 2 ? 384 : 736, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int RB = p.rows_per_cta;
-    constexpr int RPW = 16 * TPW;    // weight rows per compute warp
-    const int NW = (RB + RPW - 1) / RPW;  // compute warps
-    constexpr int CW0 = 1;           // first compute warp
+    const int NW = (RB + kRowsPerWarp - 1) / kRowsPerWarp;  // compute warps
 
     const uint32_t bars = sbase + L::BAR_OFF;
-    auto full_tma = [&](int s) { return bars + 8u * s; };
-    auto empty_smem = [&](int s) { return bars + 8u * (S + s); };
+    auto full = [&](int s) { return bars + 8u * s; };
+    auto ready = [&](int s) { return bars + 8u * (S + s); };
+    auto empty = [&](int s) { return bars + 8u * (2 * S + s); };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
-            mbar_init(full_tma(s), 1);
-            mbar_init(empty_smem(s), NW);  // every compute warp has read the stage
+            mbar_init(full(s), 1);
+            mbar_init(ready(s), 1);
+            mbar_init(empty(s), NW);  // every compute warp has read the stage
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -133,56 +211,100 @@ __global__ void __launch_bounds__(TPW == 2 ? 384 : 736, 1)
     }
     __syncthreads();
 
-    const int KS = p.K / kBKS;  // stages per chunk = scale groups
-    // Each CTA walks K from its own starting group (a multiple of the fold
-    // batch G, so that batches never wrap): the CTAs then read different x
-    // slices at any moment instead of all hitting the same L2 lines.
-    const int rot = KS % G == 0 ? (static_cast<int>(blockIdx.x) * (KS / G) / static_cast<int>(gridDim.x)) * G : 0;
-    auto kgroup = [&](int j) { return j + rot < KS ? j + rot : j + rot - KS; };
+    static_assert(S % U == 0 && (U == 2 || U == 4), "rounds tile the stage slots");
+    constexpr int RS = S / U;         // rounds per pass over the stage slots
+    const int KS = p.K / kBKS;        // scale groups = real stages per chunk
+    const int R = (KS + U - 1) / U;   // rounds per chunk
+    // Scales are read U groups at a time, as one vector load per row when
+    // every block is aligned (KS a multiple of U).
+    const bool vec_scales = KS % U == 0;
+    // Each CTA walks K from its own starting group (a multiple of U when the
+    // scale loads are vectors): the CTAs then read different x slices at any
+    // moment instead of all hitting the same L2 lines.
+    const int rot = vec_scales
+                        ? static_cast<int>(static_cast<int64_t>(blockIdx.x) * (KS / U) /
+                                           gridDim.x) * U
+                        : static_cast<int>(static_cast<int64_t>(blockIdx.x) * KS / gridDim.x);
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint32_t tx = L::X_BYTES + static_cast<uint32_t>(RB) * (kBKS / 2);
-            uint32_t it = 0;
+            uint32_t it = 0;  // stage slot = it % S, phase = (it / S) & 1
             bool ok = true;
             for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
                 const int row0 = chunk * RB;
-                for (int ks = 0; ks < KS; ++ks, ++it) {
+                int kk = rot;  // group of stage ks, rotated
+                for (int ks = 0; ks < R * U; ++ks, ++it) {
                     const int s = it % S;
-                    if (!wait_one(empty_smem(s), ((it / S) & 1u) ^ 1u, abort_flag, p.status)) {
+                    if (!wait_one(empty(s), ((it / S) & 1u) ^ 1u, abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(full_tma(s), tx);
-                    const int kk = kgroup(ks);
+                    if (ks >= KS) {  // padding stage: cycles the barrier only
+                        mbar_arrive(full(s));
+                        continue;
+                    }
+                    mbar_arrive_expect_tx(full(s), tx);
                     const uint32_t xs = sbase + L::X_OFF + s * L::X_BYTES;
-                    tma_load_2d(xs, &tmap_x, full_tma(s), kk * kBKS, 0);
-                    tma_load_2d(xs + L::X_BOX, &tmap_x, full_tma(s), kk * kBKS + 64, 0);
+                    tma_load_2d(xs, &tmap_x, full(s), kk * kBKS, 0);
+                    tma_load_2d(xs + L::X_BOX, &tmap_x, full(s), kk * kBKS + 64, 0);
                     const uint32_t ws = sbase + L::W_OFF + s * L::W_BYTES;
-                    tma_load_2d(ws, &tmap_w, full_tma(s), kk * (kBKS / 2), row0);
-                    tma_load_2d(ws + L::W_HALF, &tmap_w, full_tma(s), kk * (kBKS / 2),
+                    tma_load_2d(ws, &tmap_w, full(s), kk * (kBKS / 2), row0);
+                    tma_load_2d(ws + L::W_HALF, &tmap_w, full(s), kk * (kBKS / 2),
                                 row0 + RB / 2);
+                    if (++kk == KS) kk = 0;
                 }
             }
             // every load this thread issued has landed before exit
             const uint32_t last = it < static_cast<uint32_t>(S) ? it : S;
             for (uint32_t i = it - last; i < it; ++i) {
                 const uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(full_tma(i % S), (i / S) & 1u)) {
+                while (!mbar_try_wait(full(i % S), (i / S) & 1u)) {
                     if (global_timer_ns() - t0 > kWaitLimitNs) break;
                 }
             }
         }
-    } else if (warp - CW0 < NW) {
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ x reorder
+        // Every 16-byte chunk (x0..x7) of the stage's x boxes becomes
+        // (x0,x4),(x1,x5),(x2,x6),(x3,x7): the pair order of codes_signed.
+        constexpr int kChunks = L::X_BYTES / 16;
+        static_assert(kChunks % 32 == 0, "whole chunks per lane");
+        uint32_t round = 0;  // global round: slots U (round % RS) .., phase (round / RS) & 1
+        bool ok = true;
+        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+            for (int r = 0; ok && r < R; ++r, ++round) {
+                const int s0 = static_cast<int>(round % RS) * U;
+                const uint32_t ph = (round / RS) & 1u;
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int s = s0 + u;
+                    if (!wait_warp(full(s), ph, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    if (r * U + u < KS) {
+                        uint4* xs = reinterpret_cast<uint4*>(smem + L::X_OFF + s * L::X_BYTES);
+#pragma unroll
+                        for (int i = 0; i < kChunks / 32; ++i)
+                            xs[lane + 32 * i] = interleave_chunk(xs[lane + 32 * i]);
+                        // these generic writes precede the next TMA write of the slot
+                        fence_proxy_async_smem();
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(ready(s));
+                }
+            }
+        }
+    } else if (warp - kFirstComputeWarp < NW) {
         // ------------------------------------------------------------ compute warps
         // Warp cw owns local rows [32cw, 32cw+32): m16 tiles tt = 0, 1.
         // Thread (g, c): rows 32cw + 16tt + g (+8); k quad c owns k in
         // [16c, 16c+16) and [64+16c, 64+16c+16) of each 128-k stage.
-        const int cw = warp - CW0;
+        const int cw = warp - kFirstComputeWarp;
         const int g = lane >> 2;
         const int c = lane & 3;
-        const uint32_t m4 = p.m4, m8 = p.m8, m12 = p.m12;
         auto w_off = [&](int r, int piece) {
             // rows >= RB read row 0; their results are never stored
             const int rs = r < RB ? r : 0;
@@ -192,160 +314,155 @@ __global__ void __launch_bounds__(TPW == 2 ? 384 : 736, 1)
             return L::W_OFF + b * L::W_HALF + rr * (kBKS / 2) + 16 * (j ^ ((rr >> 1) & 3)) +
                    8 * (c & 1);
         };
-        int row[2 * TPW];  // rows of (tt, upper/lower half): index 2*tt + hh
-        int woff[2 * TPW][2];
+        int row[4];  // rows of (tt, upper/lower half): index 2*tt + hh
+        uint32_t wp[4][2];  // shared-memory addresses in stage slot 0
 #pragma unroll
-        for (int q = 0; q < 2 * TPW; ++q) {
-            row[q] = cw * RPW + (q >> 1) * 16 + (q & 1) * 8 + g;
-            woff[q][0] = w_off(row[q], 0);
-            woff[q][1] = w_off(row[q], 1);
+        for (int q = 0; q < 4; ++q) {
+            row[q] = cw * kRowsPerWarp + (q >> 1) * 16 + (q & 1) * 8 + g;
+            wp[q][0] = sbase + w_off(row[q], 0);
+            wp[q][1] = sbase + w_off(row[q], 1);
         }
-        uint32_t it = 0;
+        // x chunk of word i (k 64*(i>>1) + 16c + 8*(i&1) .. +8): chunk
+        // 2c + (i&1) of box i>>1, 128-byte swizzle by row g
+        uint32_t xp[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            xp[i] = sbase + L::X_OFF + g * 128 + (i >> 1) * L::X_BOX + 16 * ((2 * c + (i & 1)) ^ g);
+
+        uint32_t round = 0;
         bool ok = true;
         for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
-            int n[2 * TPW];
-            bool v[2 * TPW];
-            const uint16_t* srow[2 * TPW];
+            int n[4];
+            bool v[4];
+            const uint16_t* srow[4];
 #pragma unroll
-            for (int q = 0; q < 2 * TPW; ++q) {
+            for (int q = 0; q < 4; ++q) {
                 n[q] = chunk * RB + row[q];
                 v[q] = row[q] < RB && n[q] < p.N;
                 srow[q] = p.scales + static_cast<int64_t>(v[q] ? n[q] : 0) * KS;
             }
-            float acc[TPW][NT][4];
-            float d[G][TPW][NT][4];
-            float db[G][NT][4];  // -136 * sum x per token (same for every row)
-            uint32_t sc[2 * TPW][G];   // bf16 bits of the batch's scales, per row
-            uint32_t scn[2 * TPW][G];  // the next batch's, loaded one batch ahead
+            float acc[2][NT][4];
 #pragma unroll
-            for (int tt = 0; tt < TPW; ++tt)
+            for (int tt = 0; tt < 2; ++tt)
 #pragma unroll
                 for (int nn = 0; nn < NT; ++nn)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        acc[tt][nn][e] = 0.0f;
+                    for (int e = 0; e < 4; ++e) acc[tt][nn][e] = 0.0f;
+            // Scales as bf16 pairs: the current block of U groups and the
+            // next one, loaded U stages before use.
+            uint32_t scb[4][U / 2], scn[4][U / 2];
+            int kb = rot;  // first group of the next block
+            auto load_block = [&]() {
+                if (vec_scales) {
 #pragma unroll
-                        for (int u = 0; u < G; ++u) d[u][tt][nn][e] = 0.0f;
+                    for (int q = 0; q < 4; ++q) {
+                        if constexpr (U == 4) {
+                            const uint2 t = __ldg(reinterpret_cast<const uint2*>(srow[q] + kb));
+                            scn[q][0] = t.x;
+                            scn[q][1] = t.y;
+                        } else {
+                            scn[q][0] = __ldg(reinterpret_cast<const uint32_t*>(srow[q] + kb));
+                        }
                     }
+                    kb += U;
+                    if (kb == KS) kb = 0;
+                } else {
 #pragma unroll
-            for (int u = 0; u < G; ++u)
+                    for (int e = 0; e < U; ++e) {
 #pragma unroll
-                for (int nn = 0; nn < NT; ++nn)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) db[u][nn][e] = 0.0f;
-
-            // one 128-k stage (scale group) into accumulator set u
-            auto stage = [&](int u) -> bool {
-                const int s = it % S;
-                if (!wait_warp(full_tma(s), (it / S) & 1u, abort_flag, p.status)) return false;
-                const uint8_t* ws = smem + s * L::W_BYTES;
-                uint32_t wq[2 * TPW][4];
-#pragma unroll
-                for (int q = 0; q < 2 * TPW; ++q) {
-                    const uint2 p0 = *reinterpret_cast<const uint2*>(ws + woff[q][0]);
-                    const uint2 p1 = *reinterpret_cast<const uint2*>(ws + woff[q][1]);
-                    wq[q][0] = p0.x;
-                    wq[q][1] = p0.y;
-                    wq[q][2] = p1.x;
-                    wq[q][3] = p1.y;
+                        for (int q = 0; q < 4; ++q) {
+                            const uint32_t h = __ldg(srow[q] + kb);
+                            scn[q][e >> 1] = (e & 1) ? (scn[q][e >> 1] | (h << 16)) : h;
+                        }
+                        if (++kb == KS) kb = 0;
+                    }
                 }
-                const uint8_t* xst = smem + L::X_OFF + s * L::X_BYTES + g * 128;
+            };
+            load_block();
+
+            for (int r = 0; ok && r < R; ++r, ++round) {
+                const int s0 = static_cast<int>(round % RS) * U;
+                const uint32_t ph = (round / RS) & 1u;
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    // word i: k 64*(i>>1) + 16c + 8*(i&1) .. +8 = x chunk
-                    // 2c + (i&1) of box i>>1; it feeds two k16 steps
-                    uint4 xb[NT];
+                for (int u = 0; u < U; ++u) {
+                    const int s = s0 + u;
+                    // ready(s) completes after warp 1 has seen full(s) complete, so
+                    // the stage's TMA data is visible here too
+                    if (!wait_warp(ready(s), ph, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    if (r * U + u < KS) {
+                        if (u == 0) {
 #pragma unroll
-                    for (int nn = 0; nn < NT; ++nn)
-                        xb[nn] = interleave_chunk(*reinterpret_cast<const uint4*>(
-                            xst + (i >> 1) * L::X_BOX + nn * 8 * 128 +
-                            16 * ((2 * c + (i & 1)) ^ g)));
-                    uint32_t A[2 * TPW][4];
+                            for (int q = 0; q < 4; ++q)
 #pragma unroll
-                    for (int q = 0; q < 2 * TPW; ++q) codes_biased(wq[q][i], m4, m8, m12, A[q]);
+                                for (int e = 0; e < U / 2; ++e) scb[q][e] = scn[q][e];
+                            load_block();
+                        }
+
+                        const int wso = s * L::W_BYTES;
+                        uint32_t wq[4][4];
 #pragma unroll
-                    for (int h = 0; h < 2; ++h)
+                        for (int q = 0; q < 4; ++q) {
+                            const uint2 p0 = lds64(wp[q][0] + wso);
+                            const uint2 p1 = lds64(wp[q][1] + wso);
+                            wq[q][0] = p0.x;
+                            wq[q][1] = p0.y;
+                            wq[q][2] = p1.x;
+                            wq[q][3] = p1.y;
+                        }
+                        float d[2][NT][4];
 #pragma unroll
-                        for (int tt = 0; tt < TPW; ++tt)
+                        for (int i = 0; i < 4; ++i) {
+                            uint4 xb[NT];
 #pragma unroll
                             for (int nn = 0; nn < NT; ++nn)
-                                mma_bf16_16816(d[u][tt][nn], A[2 * tt][2 * h],
-                                               A[2 * tt + 1][2 * h], A[2 * tt][2 * h + 1],
-                                               A[2 * tt + 1][2 * h + 1],
-                                               h ? xb[nn].z : xb[nn].x,
-                                               h ? xb[nn].w : xb[nn].y);
-                    // zero point and bias: -136 * sum x for every token
-                    constexpr uint32_t kMinus136 = 0xC308C308u;
+                                xb[nn] = lds128(xp[i] + s * L::X_BYTES + nn * 8 * 128);
+                            uint32_t A[4][4];
 #pragma unroll
-                    for (int h = 0; h < 2; ++h)
+                            for (int q = 0; q < 4; ++q) codes_signed(wq[q][i], A[q]);
 #pragma unroll
-                        for (int nn = 0; nn < NT; ++nn)
-                            mma_bf16_16816(db[u][nn], kMinus136, kMinus136, kMinus136, kMinus136,
-                                           h ? xb[nn].z : xb[nn].x, h ? xb[nn].w : xb[nn].y);
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty_smem(s));
-                ++it;
-                return true;
-            };
-            // acc += s * (d - 136 * xsum) for the first `count` sets
-            auto fold = [&](int count) {
+                            for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int u = 0; u < G; ++u) {
-                    if (u >= count) break;
+                                for (int tt = 0; tt < 2; ++tt)
 #pragma unroll
-                    for (int tt = 0; tt < TPW; ++tt)
+                                    for (int nn = 0; nn < NT; ++nn) {
+                                        const uint32_t b0 = h ? xb[nn].z : xb[nn].x;
+                                        const uint32_t b1 = h ? xb[nn].w : xb[nn].y;
+                                        if (i == 0 && h == 0)
+                                            mma_bf16_16816_first(d[tt][nn], A[2 * tt][0],
+                                                                 A[2 * tt + 1][0], A[2 * tt][1],
+                                                                 A[2 * tt + 1][1], b0, b1);
+                                        else
+                                            mma_bf16_16816(d[tt][nn], A[2 * tt][2 * h],
+                                                           A[2 * tt + 1][2 * h],
+                                                           A[2 * tt][2 * h + 1],
+                                                           A[2 * tt + 1][2 * h + 1], b0, b1);
+                                    }
+                        }
+                        // acc += s * d: d0, d1 belong to the upper row, d2, d3 to the lower
 #pragma unroll
-                        for (int nn = 0; nn < NT; ++nn)
+                        for (int tt = 0; tt < 2; ++tt) {
+                            const float su = scale_at(scb[2 * tt], u);
+                            const float sl = scale_at(scb[2 * tt + 1], u);
 #pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const float corr = d[u][tt][nn][e] + db[u][nn][e];
-                                acc[tt][nn][e] = fmaf(bf16_bits_to_float(sc[2 * tt + (e >> 1)][u]),
-                                                      corr, acc[tt][nn][e]);
-                                d[u][tt][nn][e] = 0.0f;
+                            for (int nn = 0; nn < NT; ++nn) {
+                                acc[tt][nn][0] = fmaf(su, d[tt][nn][0], acc[tt][nn][0]);
+                                acc[tt][nn][1] = fmaf(su, d[tt][nn][1], acc[tt][nn][1]);
+                                acc[tt][nn][2] = fmaf(sl, d[tt][nn][2], acc[tt][nn][2]);
+                                acc[tt][nn][3] = fmaf(sl, d[tt][nn][3], acc[tt][nn][3]);
                             }
-#pragma unroll
-                    for (int nn = 0; nn < NT; ++nn)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) db[u][nn][e] = 0.0f;
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(empty(s));
                 }
-            };
-            auto load_scales = [&](int g0) {
-#pragma unroll
-                for (int q = 0; q < 2 * TPW; ++q)
-#pragma unroll
-                    for (int u = 0; u < G; ++u)
-                        scn[q][u] = (v[q] && g0 + u < KS)
-                                       ? static_cast<uint32_t>(__ldg(srow[q] + kgroup(g0 + u)))
-                                       : 0u;
-            };
-            auto take_scales = [&]() {
-#pragma unroll
-                for (int q = 0; q < 2 * TPW; ++q)
-#pragma unroll
-                    for (int u = 0; u < G; ++u) sc[q][u] = scn[q][u];
-            };
-            int ks = 0;
-            load_scales(0);
-            for (; ok && ks + G <= KS; ks += G) {
-                take_scales();
-                load_scales(ks + G);  // the next batch's, two batches before use
-#pragma unroll
-                for (int u = 0; u < G; ++u)
-                    if (!stage(u)) { ok = false; break; }
-                if (ok) fold(G);
-            }
-            if (ok && ks < KS) load_scales(ks);
-            for (; ok && ks < KS; ++ks) {  // remainder, one group at a time
-                take_scales();
-                if (ks + 1 < KS) load_scales(ks + 1);
-                if (!stage(0)) { ok = false; break; }
-                fold(1);
             }
             if (!ok) break;
             // epilogue: d0, d1 -> (upper row, tokens 2c, 2c+1); d2, d3 -> lower row
 #pragma unroll
-            for (int tt = 0; tt < TPW; ++tt)
+            for (int tt = 0; tt < 2; ++tt)
 #pragma unroll
                 for (int nn = 0; nn < NT; ++nn)
 #pragma unroll
@@ -361,15 +478,16 @@ __global__ void __launch_bounds__(TPW == 2 ? 384 : 736, 1)
     __syncthreads();
 }
 
-template <int NT, int S, int G, int TPW>
+template <int NT, int S, int U>
 cudaError_t launch_gemv_variant(const CUtensorMap* tx, const CUtensorMap* tw,
                                 const GemvParams& p, int grid, cudaStream_t stream) {
     using L = GLayout<NT, S>;
-    auto kern = w4a16_gemv_kernel<NT, S, G, TPW>;
+    auto kern = w4a16_gemv_kernel<NT, S, U>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    const int threads = 32 * (1 + (p.rows_per_cta + 16 * TPW - 1) / (16 * TPW));
+    const int threads =
+        32 * (kFirstComputeWarp + (p.rows_per_cta + kRowsPerWarp - 1) / kRowsPerWarp);
     kern<<<grid, threads, L::SMEM_BYTES, stream>>>(*tx, *tw, p);
     return cudaGetLastError();
 }
@@ -390,8 +508,10 @@ cudaError_t gemv_launch(const CUtensorMap* tx, const CUtensorMap* tw, const Gemv
                         int sm_count, cudaStream_t stream) {
     const int grid = p.num_chunks < sm_count ? p.num_chunks : sm_count;
     if (p.M <= 8)
-        return launch_gemv_variant<1, 6, W4A16_GEMV_G1, W4A16_GEMV_TPW>(tx, tw, p, grid, stream);
-    return launch_gemv_variant<2, 6, W4A16_GEMV_G2, W4A16_GEMV_TPW>(tx, tw, p, grid, stream);
+        return launch_gemv_variant<1, W4A16_GEMV_S1, W4A16_GEMV_U1>(tx, tw, p, grid, stream);
+    if (p.M <= 16)
+        return launch_gemv_variant<2, W4A16_GEMV_S2, W4A16_GEMV_U2>(tx, tw, p, grid, stream);
+    return launch_gemv_variant<4, W4A16_GEMV_S4, W4A16_GEMV_U4>(tx, tw, p, grid, stream);
 }
 
 }  // namespace w4a16

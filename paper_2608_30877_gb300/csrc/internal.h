@@ -43,9 +43,6 @@ struct GemvParams {
     int rows_per_cta;        // RB: weight rows per CTA chunk, multiple of 16, <= 384
     int num_chunks;          // ceil(N / RB)
     int nt;                  // MMA tiles per chunk: ceil(RB / 128)
-    // 2^28, 2^24, 2^20: multipliers that turn mul.hi into shifts by 4, 8, 12
-    // (run-time values so that the shifts stay on the FMA pipe)
-    uint32_t m4, m8, m12;
 };
 
 // RB for N rows spread over the SMs; tokens per tile for M.

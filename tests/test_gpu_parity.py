@@ -183,9 +183,12 @@ def test_error_codes_launch_nothing():
 @pytest.mark.parametrize("M,N,K,g", [
     (1, 1, 128, 128), (3, 100, 256, 128), (8, 1000, 1024, 128), (16, 4096, 512, 128),
     (17, 1234, 384, 128), (32, 8192, 256, 64), (32, 50000, 128, 128), (9, 77, 2048, 256),
+    (8, 60000, 640, 128), (24, 60000, 1152, 128), (2, 53600, 2176, 128),
 ])
 def test_small_m_streaming_kernel_shapes(M, N, K, g):
-    """M <= 32 with K a multiple of 128 runs the row-range streaming kernel:
-    ragged row ranges, 1-3 MMA tiles per CTA, 16 and 32 token columns."""
+    """M <= 32 with g = 128 runs the row-range streaming kernel: ragged row
+    ranges, 8, 16 and 32 token columns, group counts that leave padding stages
+    in the last round of stage slots, and N large enough that a CTA takes a
+    second row range (more row ranges than SMs)."""
     gpu, ref = _run_linear(M, N, K, g, seed=3 * M + N)
     assert_close(gpu, ref, f"{M}x{K}x{N} g{g}")
