@@ -23,10 +23,14 @@
 //     of 136 the exact q - 8 -- two integer-pipe instructions and one
 //     half-precision one per pair.  Per group the MMA sums d = sum x (q - 8)
 //     in fp32 and acc += s * d applies the scale;
-//   - the K loop is unrolled over the S stage slots, so every shared-memory
-//     address is a per-thread base plus an immediate; a chunk's stage count is
-//     padded to a multiple of S with empty stages that only cycle the
-//     barriers;
+//   - stages move in rounds of U (2 or 4): the TMA loads of a stage signal
+//     its own barrier, but warp 1 releases, and the compute warps wait for and
+//     give back, a whole round at a time, so the unrolled round body has no
+//     barrier inside it and every shared-memory address in it is a per-thread
+//     base plus an immediate.  A chunk's stage count is padded to a multiple of
+//     U with empty stages that only cycle the barriers;
+//   - scales are fetched U groups at a time (one vector load per row) a round
+//     before use;
 //   - each CTA walks K from its own starting group, so the CTAs do not all
 //     read the same x slice from L2 at the same moment.
 // Fragment k mapping: within a 128-k stage, thread quad index c owns k in
@@ -54,10 +58,10 @@
 #define W4A16_GEMV_U2 4
 #endif
 #ifndef W4A16_GEMV_S4
-#define W4A16_GEMV_S4 4
+#define W4A16_GEMV_S4 6
 #endif
 #ifndef W4A16_GEMV_U4
-#define W4A16_GEMV_U4 4
+#define W4A16_GEMV_U4 2
 #endif
 
 namespace w4a16 {
@@ -81,7 +85,9 @@ struct GLayout {
     static constexpr int X_OFF = 0;
     static constexpr int W_OFF = S * X_BYTES;
     static constexpr int BAR_OFF = W_OFF + S * W_BYTES;
-    static constexpr int NBARS = 3 * S;  // full (TMA), ready (x reordered), empty
+    // full: one per stage slot (TMA landed); ready (x reordered) and empty:
+    // one per round of stage slots
+    static constexpr int NBARS = S + 2 * (S / 2);
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;
     static_assert(X_BOX % 1024 == 0, "x boxes keep the 128-byte swizzle phase");
@@ -193,16 +199,18 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
     const int NW = (RB + kRowsPerWarp - 1) / kRowsPerWarp;  // compute warps
 
     const uint32_t bars = sbase + L::BAR_OFF;
+    static_assert(S % U == 0 && (U == 2 || U == 4), "rounds tile the stage slots");
+    constexpr int RS = S / U;  // round slots: rounds in flight
     auto full = [&](int s) { return bars + 8u * s; };
-    auto ready = [&](int s) { return bars + 8u * (S + s); };
-    auto empty = [&](int s) { return bars + 8u * (2 * S + s); };
+    auto ready = [&](int rs) { return bars + 8u * (S + rs); };
+    auto empty = [&](int rs) { return bars + 8u * (S + RS + rs); };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF);
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
-            mbar_init(full(s), 1);
-            mbar_init(ready(s), 1);
-            mbar_init(empty(s), NW);  // every compute warp has read the stage
+        for (int s = 0; s < S; ++s) mbar_init(full(s), 1);
+        for (int rs = 0; rs < RS; ++rs) {
+            mbar_init(ready(rs), 1);
+            mbar_init(empty(rs), NW);  // every compute warp has read the round
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -211,8 +219,6 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
     }
     __syncthreads();
 
-    static_assert(S % U == 0 && (U == 2 || U == 4), "rounds tile the stage slots");
-    constexpr int RS = S / U;         // rounds per pass over the stage slots
     const int KS = p.K / kBKS;        // scale groups = real stages per chunk
     const int R = (KS + U - 1) / U;   // rounds per chunk
     // Scales are read U groups at a time, as one vector load per row when
@@ -237,7 +243,9 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
                 int kk = rot;  // group of stage ks, rotated
                 for (int ks = 0; ks < R * U; ++ks, ++it) {
                     const int s = it % S;
-                    if (!wait_one(empty(s), ((it / S) & 1u) ^ 1u, abort_flag, p.status)) {
+                    // a round's slots are refilled once every compute warp has left it
+                    if (s % U == 0 &&
+                        !wait_one(empty(s / U), ((it / S) & 1u) ^ 1u, abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
@@ -289,22 +297,28 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 #pragma unroll
                         for (int i = 0; i < kChunks / 32; ++i)
                             xs[lane + 32 * i] = interleave_chunk(xs[lane + 32 * i]);
-                        // these generic writes precede the next TMA write of the slot
-                        fence_proxy_async_smem();
                     }
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(ready(s));
                 }
+                if (!ok) break;
+                // these generic writes precede the next TMA writes of the slots
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(ready(s0 / U));
             }
         }
     } else if (warp - kFirstComputeWarp < NW) {
         // ------------------------------------------------------------ compute warps
         // Warp cw owns local rows [32cw, 32cw+32): m16 tiles tt = 0, 1.
-        // Thread (g, c): rows 32cw + 16tt + g (+8); k quad c owns k in
-        // [16c, 16c+16) and [64+16c, 64+16c+16) of each 128-k stage.
+        // Thread (g, c): fragment rows g and g + 8 of tiles tt = 0, 1; k quad
+        // c owns k in [16c, 16c+16) and [64+16c, 64+16c+16) of each 128-k
+        // stage.  Fragment row g holds weight row 32cw + 16tt + gr (+8), with
+        // gr = g with bits 1 and 2 swapped: the four rows a half warp reads
+        // in one 8-byte load are then 0, 1, 4, 5 (or 2, 3, 6, 7) of an 8-row
+        // group, which the 64-byte swizzle puts on distinct banks.
         const int cw = warp - kFirstComputeWarp;
         const int g = lane >> 2;
         const int c = lane & 3;
+        const int gr = (g & 1) | ((g & 2) << 1) | ((g & 4) >> 1);
         auto w_off = [&](int r, int piece) {
             // rows >= RB read row 0; their results are never stored
             const int rs = r < RB ? r : 0;
@@ -318,7 +332,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
         uint32_t wp[4][2];  // shared-memory addresses in stage slot 0
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            row[q] = cw * kRowsPerWarp + (q >> 1) * 16 + (q & 1) * 8 + g;
+            row[q] = cw * kRowsPerWarp + (q >> 1) * 16 + (q & 1) * 8 + gr;
             wp[q][0] = sbase + w_off(row[q], 0);
             wp[q][1] = sbase + w_off(row[q], 1);
         }
@@ -351,6 +365,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
             // Scales as bf16 pairs: the current block of U groups and the
             // next one, loaded U stages before use.
             uint32_t scb[4][U / 2], scn[4][U / 2];
+
             int kb = rot;  // first group of the next block
             auto load_block = [&]() {
                 if (vec_scales) {
@@ -383,15 +398,15 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
             for (int r = 0; ok && r < R; ++r, ++round) {
                 const int s0 = static_cast<int>(round % RS) * U;
                 const uint32_t ph = (round / RS) & 1u;
+                // ready completes after warp 1 has seen every full(s) of the
+                // round complete, so the stages' TMA data is visible here too
+                if (!wait_warp(ready(s0 / U), ph, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
 #pragma unroll
                 for (int u = 0; u < U; ++u) {
                     const int s = s0 + u;
-                    // ready(s) completes after warp 1 has seen full(s) complete, so
-                    // the stage's TMA data is visible here too
-                    if (!wait_warp(ready(s), ph, abort_flag, p.status)) {
-                        ok = false;
-                        break;
-                    }
                     if (r * U + u < KS) {
                         if (u == 0) {
 #pragma unroll
@@ -455,9 +470,9 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
                             }
                         }
                     }
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(empty(s));
                 }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty(s0 / U));
             }
             if (!ok) break;
             // epilogue: d0, d1 -> (upper row, tokens 2c, 2c+1); d2, d3 -> lower row
