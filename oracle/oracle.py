@@ -56,6 +56,7 @@ def lib():
         L.oracle_dequant.argtypes = [p, p, i64, i64, i64, p]
         L.oracle_linear_rows.argtypes = [p, p, p, i64, i64, i64, i64, p, i64, p, ctypes.c_int]
         L.oracle_linear_points.argtypes = [p, p, p, i64, i64, i64, i64, p, p, i64, p, ctypes.c_int]
+        L.oracle_epilogue_rows.argtypes = [p, i64, i64, p, p, p, ctypes.c_int, p]
         L.oracle_max_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -145,6 +146,26 @@ def linear_points(x_bits: np.ndarray, packed: np.ndarray, scales: np.ndarray,
     out = np.empty(mi.shape[0], dtype=np.float64)
     lib().oracle_linear_points(_ptr(x_bits), _ptr(packed), _ptr(scales), M, N, K, g,
                                _ptr(mi), _ptr(ni), mi.shape[0], _ptr(out), int(nthreads))
+    return out
+
+
+ACT_NONE, ACT_SWIGLU, ACT_GELU = 0, 1, 2
+
+
+def epilogue_rows(y: np.ndarray, act: int = ACT_NONE, bias=None, residual=None,
+                  rows=None) -> np.ndarray:
+    """Fused epilogue on fp64 linear outputs y [nrows, N] (rows `rows` of the
+    batch): act(y + bias) + residual, fp64 [nrows, N_out]; SwiGLU takes rows
+    (2j, 2j+1) of the weights as (gate, up) of output j."""
+    y = np.ascontiguousarray(y, dtype=np.float64)
+    nrows, N = y.shape
+    rows = np.arange(nrows, dtype=np.int64) if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    n_out = N // 2 if act == ACT_SWIGLU else N
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.uint16)
+    res = None if residual is None else np.ascontiguousarray(residual, dtype=np.uint16)
+    out = np.empty((nrows, n_out), dtype=np.float64)
+    lib().oracle_epilogue_rows(_ptr(y), nrows, N, None if b is None else _ptr(b),
+                               None if res is None else _ptr(res), _ptr(rows), int(act), _ptr(out))
     return out
 
 

@@ -187,6 +187,44 @@ void oracle_linear_points(const uint16_t* x, const uint8_t* packed,
     (void)nthreads;
 }
 
+/* ---- fused epilogue --------------------------------------------------------
+ *
+ * Operator fusion of what follows a linear layer into its output stage -- the
+ * optimisation the paper names as future work (Sec. 5).  The paper names no
+ * activation; the readings fixed for this library are the usual decoder ones:
+ *   z[n]   = y[n] + bias[n]                       (bias optional, bf16 [N])
+ *   act 0: h[n] = z[n]                            (N_out = N)
+ *   act 1: SwiGLU over interleaved rows: h[j] = silu(z[2j]) * z[2j+1],
+ *          silu(t) = t / (1 + exp(-t))            (N_out = N / 2)
+ *   act 2: GELU, h[n] = z[n] * Phi(z[n]) = z/2 * (1 + erf(z / sqrt 2))
+ *   out[j] = h[j] + residual[m, j]                (residual optional, bf16
+ *                                                  [M, N_out])
+ * all in fp64.  y: fp64 [nrows, N] for the rows `rows` of the batch. */
+static double silu_d(double t) { return t / (1.0 + exp(-t)); }
+static double gelu_d(double t) { return 0.5 * t * (1.0 + erf(t / sqrt(2.0))); }
+
+void oracle_epilogue_rows(const double* y, int64_t nrows, int64_t N, const uint16_t* bias,
+                          const uint16_t* residual, const int64_t* rows, int act,
+                          double* out) {
+    int64_t n_out = act == 1 ? N / 2 : N;
+    for (int64_t r = 0; r < nrows; ++r) {
+        const double* yr = y + r * N;
+        for (int64_t j = 0; j < n_out; ++j) {
+            double h;
+            if (act == 1) {
+                double gate = yr[2 * j] + (bias ? (double)oracle_bf16_to_f32(bias[2 * j]) : 0.0);
+                double up = yr[2 * j + 1] + (bias ? (double)oracle_bf16_to_f32(bias[2 * j + 1]) : 0.0);
+                h = silu_d(gate) * up;
+            } else {
+                double z = yr[j] + (bias ? (double)oracle_bf16_to_f32(bias[j]) : 0.0);
+                h = act == 2 ? gelu_d(z) : z;
+            }
+            if (residual) h += (double)oracle_bf16_to_f32(residual[rows[r] * n_out + j]);
+            out[r * n_out + j] = h;
+        }
+    }
+}
+
 int oracle_max_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

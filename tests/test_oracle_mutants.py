@@ -2,7 +2,9 @@
 
 Each case compiles a copy of oracle/w4a16_oracle.c with one planted mistake
 (swapped nibbles, dropped zero point, wrong group index, round-half-away,
-truncating bf16 rounding, fp32 accumulation, wrong activation row), points
+truncating bf16 rounding, fp32 accumulation, wrong activation row, and in
+the fused epilogue swapped gate/up, a wrong SiLU sign, the tanh GELU
+approximation, a wrong residual row, bias after the activation), points
 the oracle module at it and runs the pins: at least one must fail.  The
 mistakes live only in temporary copies on the CPU."""
 import ctypes
@@ -25,6 +27,13 @@ MUTANTS = {
     "bf16_truncates": [("u += 0x7FFFu + kept_lsb;", "u += 0u * kept_lsb;")],
     "fp32_accumulate": [("double acc = 0.0;", "float acc = 0.0f;")],
     "wrong_x_row": [("const uint16_t* xrow = x + rows[r] * K;", "const uint16_t* xrow = x;")],
+    "swiglu_gate_up_swapped": [("h = silu_d(gate) * up;", "h = silu_d(up) * gate;")],
+    "silu_wrong_sign": [("return t / (1.0 + exp(-t));", "return t / (1.0 + exp(t));")],
+    "gelu_tanh_approximation": [("return 0.5 * t * (1.0 + erf(t / sqrt(2.0)));",
+                                 "return 0.5 * t * (1.0 + tanh(0.7978845608028654 * (t + 0.044715 * t * t * t)));")],
+    "residual_wrong_row": [("residual[rows[r] * n_out + j]", "residual[r * n_out + j]")],
+    "bias_after_activation": [("h = act == 2 ? gelu_d(z) : z;",
+                               "h = act == 2 ? gelu_d(yr[j]) + (z - yr[j]) : z;")],
 }
 
 PINS = [
@@ -40,6 +49,11 @@ PINS = [
     P.test_quantize_hand_example,
     P.test_quantize_rounds_half_to_even_and_zero_group,
     P.test_quantize_error_bound_and_code_range,
+    P.test_epilogue_silu_closed_form,
+    P.test_epilogue_swiglu_hand_example_and_gate_up_order,
+    P.test_epilogue_gelu_normal_cdf_values,
+    P.test_epilogue_bias_residual_by_hand,
+    P.test_epilogue_bias_enters_before_the_activation,
 ]
 
 
@@ -64,7 +78,7 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
         mut = ctypes.CDLL(so)
         for fn in ("oracle_bf16_rne", "oracle_bf16_to_f32", "oracle_unpack", "oracle_pack",
                    "oracle_quantize", "oracle_dequant", "oracle_linear_rows",
-                   "oracle_linear_points", "oracle_max_threads"):
+                   "oracle_linear_points", "oracle_epilogue_rows", "oracle_max_threads"):
             getattr(mut, fn).argtypes = getattr(good, fn).argtypes
             getattr(mut, fn).restype = getattr(good, fn).restype
         monkeypatch.setattr(O, "_lib", mut)

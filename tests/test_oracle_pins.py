@@ -297,3 +297,55 @@ def test_error_metrics():
     assert abs(m["rms_ref"] - math.sqrt(12.5)) < 1e-12
     assert abs(m["max_abs_err"] - 0.1) < 1e-12
     assert abs(m["rel_fro"] - 0.1 / 5.0) < 1e-12
+
+
+# ---- fused epilogue (operator fusion, Sec. 5; activations are the library's
+# reading: SwiGLU over interleaved (gate, up) rows, exact GELU) -------------
+
+def test_epilogue_silu_closed_form():
+    # with up = 1, SwiGLU output j is silu(gate); sigma(ln 3) = 3/4, sigma(-ln 3) = 1/4
+    ln3 = math.log(3.0)
+    y = np.array([[0.0, 1.0, ln3, 1.0, -ln3, 1.0]])
+    h = O.epilogue_rows(y, O.ACT_SWIGLU)
+    assert h.shape == (1, 3)
+    assert h[0, 0] == 0.0
+    assert abs(h[0, 1] - 0.75 * ln3) < 1e-15
+    assert abs(h[0, 2] + 0.25 * ln3) < 1e-15
+
+
+def test_epilogue_swiglu_hand_example_and_gate_up_order():
+    # gate = z[2j], up = z[2j+1]: silu(ln 3) * 2 and silu(-ln 3) * 4
+    ln3 = math.log(3.0)
+    h = O.epilogue_rows(np.array([[ln3, 2.0, -ln3, 4.0]]), O.ACT_SWIGLU)
+    assert abs(h[0, 0] - 1.5 * ln3) < 1e-14
+    assert abs(h[0, 1] + 1.0 * ln3) < 1e-14
+
+
+def test_epilogue_gelu_normal_cdf_values():
+    # GELU(t) = t * Phi(t); Phi(1) = 0.841344746068542948..., Phi(-1) = 1 - Phi(1)
+    phi1 = 0.8413447460685429
+    h = O.epilogue_rows(np.array([[0.0, 1.0, -1.0, 10.0, -10.0]]), O.ACT_GELU)[0]
+    assert h[0] == 0.0
+    assert abs(h[1] - phi1) < 1e-15
+    assert abs(h[2] + (1.0 - phi1)) < 1e-15
+    assert abs(h[3] - 10.0) < 1e-12
+    assert abs(h[4]) < 1e-20
+
+
+def test_epilogue_bias_residual_by_hand():
+    # bf16 bits: 0.25 = 0x3E80, 0.5 = 0x3F00, 1.0 = 0x3F80, -1.0 = 0xBF80, 2.0 = 0x4000
+    y = np.array([[1.5, -2.0]])
+    bias = np.array([0x3E80, 0x3F00], dtype=np.uint16)
+    residual = np.array([[0x4000, 0x4000], [0x4000, 0x4000], [0x3F80, 0xBF80]], dtype=np.uint16)
+    h = O.epilogue_rows(y, O.ACT_NONE, bias=bias, residual=residual, rows=[2])
+    assert h.tolist() == [[2.75, -2.5]]            # 1.5 + 0.25 + 1, -2 + 0.5 - 1
+    assert O.epilogue_rows(y, O.ACT_NONE).tolist() == y.tolist()
+
+
+def test_epilogue_bias_enters_before_the_activation():
+    # gate 0 + bias 1 -> silu(1) = e / (1 + e); up 3 + bias 0 -> 3
+    bias = np.array([0x3F80, 0x0000], dtype=np.uint16)
+    h = O.epilogue_rows(np.array([[0.0, 3.0]]), O.ACT_SWIGLU, bias=bias)
+    assert abs(h[0, 0] - 3.0 * math.e / (1.0 + math.e)) < 1e-15
+    hg = O.epilogue_rows(np.array([[0.0]]), O.ACT_GELU, bias=np.array([0x3F80], dtype=np.uint16))
+    assert abs(hg[0, 0] - 0.8413447460685429) < 1e-15
