@@ -6,7 +6,7 @@ Default step: one pass of the 175B-class int4 linear stack -- 96 layers x
 g = 128, all ~88 GB of packed weights resident in HBM -- over a batch of 64
 protein-ligand pairs x 1024 tokens (M = 65536).  `value` is scored pairs/s.
 
-Other workloads (--config qkv | mlp_up | mlp_down | gemv | tiny) print the
+Other workloads (--config qkv | mlp_up | mlp_down | mlp_swiglu | gemv | tiny) print the
 same JSON line for one linear (TFLOP/s, or GB/s for the small-M kernel).
 
 --impl reference times the CPU oracle (the only reference there is) on a
@@ -180,9 +180,10 @@ def linear_flops(M, N, K):
     return 2.0 * M * N * K
 
 
-def linear_bytes(M, N, K, g):
+def linear_bytes(M, N, K, g, n_out=None):
     """Algorithmic bytes of one linear: packed weights + scales + x once + out once."""
-    return N * K / 2 + 2.0 * N * (K // g) + 2.0 * M * K + 2.0 * M * N
+    n_out = N if n_out is None else n_out
+    return N * K / 2 + 2.0 * N * (K // g) + 2.0 * M * K + 2.0 * M * n_out
 
 
 def make_weights(N, K, g, seed):
@@ -253,15 +254,16 @@ class LinearWorkload:
     """One linear shape; for the small-M kernel the weights rotate over copies
     so that no launch finds its weights in L2."""
 
-    def __init__(self, name, M, N, K, g, seed, copies=1):
+    def __init__(self, name, M, N, K, g, seed, copies=1, act=0):
         import torch
         from paper_2608_30877_gb300 import synthetic as S
-        self.name, self.M, self.N, self.K, self.g = name, M, N, K, g
+        self.name, self.M, self.N, self.K, self.g, self.act = name, M, N, K, g, act
         self.x = S.make_x(M, K, seed, "cuda")
-        self.out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        n_out = N // 2 if act == 1 else N
+        self.out = torch.empty((M, n_out), dtype=torch.bfloat16, device="cuda")
         self.w = [make_weights(N, K, g, seed + 10 * c) for c in range(copies)]
         self.flops = linear_flops(M, N, K)
-        self.bytes = linear_bytes(M, N, K, g)
+        self.bytes = linear_bytes(M, N, K, g, n_out)
         self.launches_per_step = 1
         self.i = 0
 
@@ -269,7 +271,11 @@ class LinearWorkload:
         from paper_2608_30877_gb300 import w4a16 as W
         packed, scales = self.w[self.i % len(self.w)]
         self.i += 1
-        W.linear(self.x, packed, scales, self.g, out=self.out, stream=stream)
+        if self.act:
+            W.linear_fused(self.x, packed, scales, self.g, act=self.act, out=self.out,
+                           stream=stream)
+        else:
+            W.linear(self.x, packed, scales, self.g, out=self.out, stream=stream)
 
 
 # ----------------------------------------------------------------- CPU oracle
@@ -316,14 +322,18 @@ def config_for(args):
                 "pairs": args.pairs, "tokens_per_pair": 1024, "layers": args.layers, "g": 128,
                 "l2": "inputs larger than L2 (88 GB packed weights, >=1.6 GB activations per "
                       "linear); no flush"}
-    cases = {"qkv": S.QKV_PREFILL, "mlp_up": S.MLP_UP, "mlp_down": S.MLP_DOWN, "tiny": S.TINY}
+    cases = {"qkv": S.QKV_PREFILL, "mlp_up": S.MLP_UP, "mlp_down": S.MLP_DOWN, "tiny": S.TINY,
+             "mlp_swiglu": S.MLP_SWIGLU}
     if c == "gemv":
         lc = S.gemv_case(args.m)
     else:
         lc = cases[c]
-    return {"workload": lc.name, "M": lc.M, "N": lc.N, "K": lc.K, "g": lc.g,
-            "l2": "weights rotate over 2 copies larger than L2" if c == "gemv"
-            else "inputs larger than L2; no flush"}
+    cfg = {"workload": lc.name, "M": lc.M, "N": lc.N, "K": lc.K, "g": lc.g,
+           "l2": "weights rotate over 2 copies larger than L2" if c == "gemv"
+           else "inputs larger than L2; no flush"}
+    if c == "mlp_swiglu":
+        cfg["epilogue"] = "SwiGLU over interleaved gate/up rows, output N/2 columns"
+    return cfg
 
 
 def run_reference(args):
@@ -367,7 +377,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="stack",
-                    choices=["stack", "qkv", "mlp_up", "mlp_down", "gemv", "tiny"])
+                    choices=["stack", "qkv", "mlp_up", "mlp_down", "mlp_swiglu", "gemv", "tiny"])
     ap.add_argument("--m", type=int, default=32, help="tokens for --config gemv")
     ap.add_argument("--pairs", type=int, default=64)
     ap.add_argument("--layers", type=int, default=96)
@@ -397,7 +407,8 @@ def main():
         from paper_2608_30877_gb300 import synthetic as S
         cfg = config_for(args)
         copies = 2 if args.config == "gemv" else 1
-        wl = LinearWorkload(cfg["workload"], cfg["M"], cfg["N"], cfg["K"], cfg["g"], 3, copies)
+        wl = LinearWorkload(cfg["workload"], cfg["M"], cfg["N"], cfg["K"], cfg["g"], 3, copies,
+                            act=1 if args.config == "mlp_swiglu" else 0)
         unit = "GB/s" if args.config == "gemv" else "TFLOP/s"
         units_per_step = None
     setup_s = time.perf_counter() - setup_t0

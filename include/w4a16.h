@@ -78,6 +78,41 @@ int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales
                  void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,
                  void* stream);
 
+/* Activation of the fused epilogue (w4a16_linear_fused). */
+typedef enum {
+    W4A16_ACT_NONE = 0,
+    /* SwiGLU over interleaved rows: rows 2j and 2j+1 of the weights are the
+     * gate and up projections of output column j; h[m,j] = silu(z[m,2j]) *
+     * z[m,2j+1] with silu(t) = t / (1 + e^-t).  N must be even; the output
+     * has N/2 columns. */
+    W4A16_ACT_SWIGLU = 1,
+    /* GELU, exact form: h = z * Phi(z) = z/2 * (1 + erf(z / sqrt 2)). */
+    W4A16_ACT_GELU = 2
+} w4a16_activation;
+
+/*
+ * out = act(x * dequant(w_packed, scales)^T + bias) + residual: the linear
+ * layer with what follows it fused into its output stage -- the operator
+ * fusion the paper names as the next optimisation (Sec. 5).  The paper names
+ * no activation; SwiGLU and GELU are the usual decoder ones.
+ *   x, w_packed, scales, M, N, K, g   as in w4a16_linear
+ *   bias_bf16      [N] bf16, device, added to every row before the
+ *                  activation; NULL for none
+ *   residual_bf16  [M, N_out] bf16, device, added after the activation; NULL
+ *                  for none.  It may be out itself (in-place residual add);
+ *                  otherwise it must not overlap out.
+ *   out_bf16       [M, N_out] bf16, device: N_out = N/2 for SwiGLU, else N
+ *   activation     a w4a16_activation (else W4A16_ERR_INVALID_ARG; SwiGLU
+ *                  with odd N is W4A16_ERR_INVALID_ARG)
+ * Everything after the fp32 accumulation is computed in fp32 with one bf16
+ * rounding at the store.  Pointers follow the 16-byte rule.  With
+ * activation NONE and both pointers NULL this is w4a16_linear.
+ */
+int w4a16_linear_fused(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
+                       const void* bias_bf16, const void* residual_bf16, void* out_bf16,
+                       int64_t M, int64_t N, int64_t K, int64_t g, int activation,
+                       void* stream);
+
 /* One int4 linear layer of a stack.  The caller owns every pointer. */
 typedef struct {
     const void* x;          /* bf16 [M, K] */

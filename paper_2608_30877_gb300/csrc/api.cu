@@ -130,6 +130,37 @@ int check_linear(const void* x, const void* w, const void* s, const void* out, i
     return W4A16_OK;
 }
 
+Epilogue plain_epilogue(int64_t N) { return Epilogue{nullptr, nullptr, 0, static_cast<int>(N)}; }
+
+// Arguments of w4a16_linear_fused beyond those of w4a16_linear.
+int check_fused(const void* x, const void* w, const void* s, const void* bias,
+                const void* residual, const void* out, int64_t M, int64_t N, int64_t K,
+                int64_t g, int act) {
+    if (act != W4A16_ACT_NONE && act != W4A16_ACT_SWIGLU && act != W4A16_ACT_GELU)
+        return W4A16_ERR_INVALID_ARG;
+    if (act == W4A16_ACT_SWIGLU && N % 2 != 0) return W4A16_ERR_INVALID_ARG;
+    const int64_t n_out = act == W4A16_ACT_SWIGLU ? N / 2 : N;
+    if (x == nullptr || out == nullptr) return W4A16_ERR_INVALID_ARG;
+    if (M <= 0) return W4A16_ERR_INVALID_ARG;
+    int rc = check_weights(w, s, N, K, g);
+    if (rc != W4A16_OK) return rc;
+    if (M > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(x) || !aligned16(out)) return W4A16_ERR_ALIGNMENT;
+    if ((bias != nullptr && !aligned16(bias)) || (residual != nullptr && !aligned16(residual)))
+        return W4A16_ERR_ALIGNMENT;
+    const int64_t out_bytes = M * n_out * 2;
+    if (overlaps(out, out_bytes, x, M * K * 2) || overlaps(out, out_bytes, w, N * (K / 2)) ||
+        overlaps(out, out_bytes, s, N * (K / g) * 2) ||
+        (bias != nullptr && overlaps(out, out_bytes, bias, N * 2)))
+        return W4A16_ERR_INVALID_ARG;
+    // the residual is read where out is written: the same buffer, or disjoint
+    if (residual != nullptr && residual != out && overlaps(out, out_bytes, residual, out_bytes))
+        return W4A16_ERR_INVALID_ARG;
+    const int64_t tiles = ((M + 31) / 32) * ((N + 127) / 128);
+    if (tiles > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    return W4A16_OK;
+}
+
 int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uint64_t inner,
               uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
               CUtensorMapSwizzle swz) {
@@ -147,7 +178,8 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
 // M <= 32 with g = 128: the streaming kernel (rows spread evenly over the
 // SMs).
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
-                int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
+                int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
+                cudaStream_t stream) {
     const int T = gemv_tokens_per_tile(M);
     const int RB = gemv_rows_per_cta(N, st.sm_count);
     alignas(64) CUtensorMap tx;
@@ -169,15 +201,17 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
     p.rows_per_cta = RB;
     p.num_chunks = static_cast<int>((N + RB - 1) / RB);
     p.nt = (RB + 127) / 128;
+    p.epi = epi;
     return gemv_launch(&tx, &tw, p, st.sm_count, stream) == cudaSuccess ? W4A16_OK
                                                                          : W4A16_ERR_CUDA;
 }
 
 // Validated arguments -> one kernel launch.
 int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
-                  int64_t M, int64_t N, int64_t K, int64_t g, cudaStream_t stream) {
+                  int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
+                  cudaStream_t stream) {
     if (M <= 32 && g == 128 && K % 128 == 0 && g_small_m_streaming)
-        return launch_gemv(st, x, w, s, out, M, N, K, g, stream);
+        return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
     alignas(64) CUtensorMap tx;
@@ -200,6 +234,7 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     p.num_w_tiles = static_cast<int>((N + 127) / 128);
     p.num_tiles = p.num_t_tiles * p.num_w_tiles;
     p.group_t = v == TsVariant::kGemm256 ? g_group_t : 1;
+    p.epi = epi;
     const int grid = ts_grid(v, p, st.sm_count);
     return ts_launch(v, &tx, &tw, p, grid, stream) == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
 }
@@ -218,6 +253,23 @@ extern "C" int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const v
     rc = device_state(&st);
     if (rc != W4A16_OK) return rc;
     return launch_linear(*st, x_bf16, w_packed_u8, scales_bf16, out_bf16, M, N, K, g,
+                         plain_epilogue(N), static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int w4a16_linear_fused(const void* x_bf16, const void* w_packed_u8,
+                                  const void* scales_bf16, const void* bias_bf16,
+                                  const void* residual_bf16, void* out_bf16, int64_t M, int64_t N,
+                                  int64_t K, int64_t g, int activation, void* stream) {
+    int rc = check_fused(x_bf16, w_packed_u8, scales_bf16, bias_bf16, residual_bf16, out_bf16, M,
+                         N, K, g, activation);
+    if (rc != W4A16_OK) return rc;
+    DeviceState* st = nullptr;
+    rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    const Epilogue epi{static_cast<const uint16_t*>(bias_bf16),
+                       static_cast<const uint16_t*>(residual_bf16), activation,
+                       static_cast<int>(activation == W4A16_ACT_SWIGLU ? N / 2 : N)};
+    return launch_linear(*st, x_bf16, w_packed_u8, scales_bf16, out_bf16, M, N, K, g, epi,
                          static_cast<cudaStream_t>(stream));
 }
 
@@ -235,7 +287,7 @@ extern "C" int w4a16_linear_stack(const w4a16_layer* layers, int64_t n_layers, i
     for (int64_t i = 0; i < n_layers; ++i) {
         const w4a16_layer& l = layers[i];
         rc = launch_linear(*st, l.x, l.w_packed, l.scales, l.out, M, l.N, l.K, g,
-                           static_cast<cudaStream_t>(stream));
+                           plain_epilogue(l.N), static_cast<cudaStream_t>(stream));
         if (rc != W4A16_OK) return rc;
     }
     return W4A16_OK;
@@ -317,4 +369,4 @@ extern "C" const char* w4a16_status_string(int status) {
     }
 }
 
-extern "C" int w4a16_version(void) { return 100; }
+extern "C" int w4a16_version(void) { return 200; }

@@ -39,6 +39,7 @@
 // Every wait is bounded (ptx.cuh): on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, drains its copies and returns.
 #include "dequant.cuh"
+#include "epilogue.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -182,8 +183,8 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 // NT: 8-token MMA column tiles (T = 8 NT staged token rows); S: stage slots;
 // U: stages per unrolled round of the K loop, and scale groups per load (a
-// divisor of S).
-template <int NT, int S, int U>
+// divisor of S); FUSED: the fused epilogue (bias, activation, residual).
+template <int NT, int S, int U, bool FUSED>
 __global__ void __launch_bounds__(kMaxThreads, 1)
     w4a16_gemv_kernel(const __grid_constant__ CUtensorMap tmap_x,
                       const __grid_constant__ CUtensorMap tmap_w, const GemvParams p) {
@@ -476,18 +477,53 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
             }
             if (!ok) break;
             // epilogue: d0, d1 -> (upper row, tokens 2c, 2c+1); d2, d3 -> lower row
+            const Epilogue& ep = p.epi;
+            if constexpr (!FUSED) {
 #pragma unroll
-            for (int tt = 0; tt < 2; ++tt)
+                for (int tt = 0; tt < 2; ++tt)
 #pragma unroll
-                for (int nn = 0; nn < NT; ++nn)
+                    for (int nn = 0; nn < NT; ++nn)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int q = 2 * tt + (e >> 1);
-                        const int m = nn * 8 + 2 * c + (e & 1);
-                        if (v[q] && m < p.M)
-                            p.out[static_cast<int64_t>(m) * p.N + n[q]] =
-                                __bfloat16_as_ushort(__float2bfloat16_rn(acc[tt][nn][e]));
-                    }
+                        for (int e = 0; e < 4; ++e) {
+                            const int q = 2 * tt + (e >> 1);
+                            const int m = nn * 8 + 2 * c + (e & 1);
+                            if (v[q] && m < p.M)
+                                p.out[static_cast<int64_t>(m) * p.N + n[q]] =
+                                    __bfloat16_as_ushort(__float2bfloat16_rn(acc[tt][nn][e]));
+                        }
+            } else {
+                // Fused epilogue.  A row's parity is that of g (the row remap
+                // keeps bit 0), so SwiGLU's partner row n ^ 1 is held by lane
+                // ^ 4 with the same tokens; the gate (even-row) lane finishes.
+                float bq[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    bq[q] = (ep.bias != nullptr && v[q]) ? bf16_to_f32(ep.bias[n[q]]) : 0.0f;
+#pragma unroll
+                for (int tt = 0; tt < 2; ++tt)
+#pragma unroll
+                    for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int q = 2 * tt + (e >> 1);
+                            const int m = nn * 8 + 2 * c + (e & 1);
+                            const float z = acc[tt][nn][e] + bq[q];
+                            if (ep.act == kActSwiGLU) {
+                                const float up = __shfl_xor_sync(0xffffffffu, z, 4);
+                                if ((g & 1) == 0 && v[q] && m < p.M) {
+                                    const int64_t o = static_cast<int64_t>(m) * ep.n_out + (n[q] >> 1);
+                                    float h = silu_f32(z) * up;
+                                    if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                                    p.out[o] = f32_to_bf16_rn(h);
+                                }
+                            } else if (v[q] && m < p.M) {
+                                const int64_t o = static_cast<int64_t>(m) * ep.n_out + n[q];
+                                float h = ep.act == kActGELU ? gelu_f32(z) : z;
+                                if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                                p.out[o] = f32_to_bf16_rn(h);
+                            }
+                        }
+            }
         }
     }
     __syncthreads();
@@ -497,7 +533,10 @@ template <int NT, int S, int U>
 cudaError_t launch_gemv_variant(const CUtensorMap* tx, const CUtensorMap* tw,
                                 const GemvParams& p, int grid, cudaStream_t stream) {
     using L = GLayout<NT, S>;
-    auto kern = w4a16_gemv_kernel<NT, S, U>;
+    // the plain variant keeps the fused epilogue's registers out of the K loop
+    const bool fused =
+        p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
+    auto kern = fused ? w4a16_gemv_kernel<NT, S, U, true> : w4a16_gemv_kernel<NT, S, U, false>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;

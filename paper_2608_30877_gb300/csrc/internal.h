@@ -8,6 +8,16 @@
 
 namespace w4a16 {
 
+// Fused epilogue of a linear layer: out = act(acc + bias) + residual, with
+// act one of none, SwiGLU over interleaved (gate, up) rows (n_out = N / 2)
+// or GELU.  All pointers are bf16 bits; null means absent.
+struct Epilogue {
+    const uint16_t* bias;      // [N]
+    const uint16_t* residual;  // [M, n_out]; may be the output itself
+    int act;                   // 0 none, 1 SwiGLU, 2 GELU (the ABI's w4a16_activation)
+    int n_out;                 // output columns: N, or N / 2 for SwiGLU
+};
+
 // Parameters of the fused dequant + tcgen05 kernel (everything except the
 // two TMA descriptors, which are passed as __grid_constant__ arguments).
 struct TsParams {
@@ -19,6 +29,7 @@ struct TsParams {
     int num_w_tiles;         // weight tiles: ceil(N / 128)
     int num_tiles;
     int group_t;             // raster: token tiles per group
+    Epilogue epi;
 };
 
 // Kernel variants of the fused kernel.  Both take 128 weight rows per tile
@@ -43,6 +54,7 @@ struct GemvParams {
     int rows_per_cta;        // RB: weight rows per CTA chunk, multiple of 16, <= 384
     int num_chunks;          // ceil(N / RB)
     int nt;                  // MMA tiles per chunk: ceil(RB / 128)
+    Epilogue epi;
 };
 
 // RB for N rows spread over the SMs; tokens per tile for M.

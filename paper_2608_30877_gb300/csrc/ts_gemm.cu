@@ -12,7 +12,7 @@
 // bf16 weight tile never touches shared memory, which keeps shared-memory
 // bandwidth for the x tiles the MMA reads.
 //
-// Warp roles (32 * (6 + 4*DQ) threads):
+// Warp roles (32 * (2 + 4*DQ + 4*EP) threads):
 //   warp 0      TMA producer: x tile [T x 64] and packed weight tile [128 x 32 B]
 //               per stage into a ring of S_SMEM shared-memory stages;
 //   warp 1      allocates tensor memory, one thread issues the MMAs;
@@ -20,8 +20,11 @@
 //               thread = one weight row (its TMEM lane), 32 packed bytes ->
 //               64 bf16 -> 32 TMEM columns per stage, into a ring of S_TMEM
 //               tensor-memory A stages;
-//   last 4      epilogue: tcgen05.ld of the accumulator, fp32 -> bf16,
-//               stores to out.
+//   last 4*EP   epilogue, EP groups of four warps splitting the tile's
+//               32-token chunks: tcgen05.ld of the accumulator, the fused
+//               epilogue if any (bias, activation, residual), fp32 -> bf16,
+//               stores to out.  The next tile's MMAs wait until the
+//               accumulator is drained, so two groups halve that wait.
 // A warp may only touch the 32 TMEM lanes of its sub-partition (warp % 4), so
 // each group of four warps covers all 128 lanes.
 //
@@ -29,6 +32,7 @@
 // W4A16_ERR_TIMEOUT, drains its own copies and MMAs, frees tensor memory and
 // returns.
 #include "dequant.cuh"
+#include "epilogue.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -85,13 +89,153 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return r;
 }
 
-template <int DQ>
-constexpr int threads_for() {
-    return 32 * (6 + 4 * DQ);
+// Fused epilogue of one tile for the epilogue thread that owns weight row n
+// (TMEM lane `lane` of its sub-partition): the 32-token chunks c0, c0 + cs,
+// ... of the T tokens from TMEM column d_col.  Residuals of a chunk are read
+// before any of its outputs is written (the residual may be the output).
+// SwiGLU pairs rows (n, n ^ 1) = (gate, up) of output column n / 2 across
+// neighbouring lanes: the even lane finishes the even tokens, the odd lane
+// the odd ones.  Otherwise neighbouring lanes swap values so that each store
+// writes the outputs (n, n+1) of one token as a 32-bit word (even n_out).
+template <int T>
+__device__ __forceinline__ void fused_epilogue_tile(const TsParams& p, uint32_t d_col, int m0,
+                                                    int n, int lane, int c0, int cs) {
+    const Epilogue& e = p.epi;
+    const bool n_ok = n < p.N;
+    const bool has_res = e.residual != nullptr;
+    const float b = (e.bias != nullptr && n_ok) ? bf16_to_f32(e.bias[n]) : 0.0f;
+    const bool odd = (lane & 1) != 0;
+#pragma unroll 1
+    for (int c = c0; c < T / 32; c += cs) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(d_col + c * 32, v);
+        tmem_ld_wait(v);
+        const int mbase = m0 + c * 32;
+        if (e.act == kActSwiGLU) {
+            const int col = n >> 1;
+            float r[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int m = mbase + 2 * j + (odd ? 1 : 0);
+                r[j] = (has_res && m < p.M && n_ok)
+                           ? bf16_to_f32(e.residual[static_cast<int64_t>(m) * e.n_out + col])
+                           : 0.0f;
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float z0 = __uint_as_float(v[2 * j]) + b;
+                const float z1 = __uint_as_float(v[2 * j + 1]) + b;
+                const float other = __shfl_xor_sync(0xffffffffu, odd ? z0 : z1, 1);
+                const int m = mbase + 2 * j + (odd ? 1 : 0);
+                const float h = (odd ? silu_f32(other) * z1 : silu_f32(z0) * other) + r[j];
+                if (m < p.M && n_ok) p.out[static_cast<int64_t>(m) * e.n_out + col] = f32_to_bf16_rn(h);
+            }
+        } else if ((e.n_out & 1) == 0) {
+            // even lane: token 2j, columns (n, n+1); odd lane: token 2j+1, (n-1, n)
+            const int col = odd ? n - 1 : n;
+            uint32_t rw[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int m = mbase + 2 * j + (odd ? 1 : 0);
+                rw[j] = (has_res && m < p.M && n_ok)
+                            ? *reinterpret_cast<const uint32_t*>(
+                                  e.residual + static_cast<int64_t>(m) * e.n_out + col)
+                            : 0u;
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                float h0 = __uint_as_float(v[2 * j]) + b, h1 = __uint_as_float(v[2 * j + 1]) + b;
+                if (e.act == kActGELU) {
+                    h0 = gelu_f32(h0);
+                    h1 = gelu_f32(h1);
+                }
+                const float other = __shfl_xor_sync(0xffffffffu, odd ? h0 : h1, 1);
+                const int m = mbase + 2 * j + (odd ? 1 : 0);
+                // (lo, hi) = outputs (col, col + 1) of token m
+                float lo = odd ? other : h0, hi = odd ? h1 : other;
+                lo += __uint_as_float(rw[j] << 16);
+                hi += __uint_as_float(rw[j] & 0xFFFF0000u);
+                if (m < p.M && n_ok)
+                    *reinterpret_cast<uint32_t*>(p.out + static_cast<int64_t>(m) * e.n_out + col) =
+                        pack_bf16x2(lo, hi);
+            }
+        } else {
+            float r[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const int m = mbase + j;
+                r[j] = (has_res && m < p.M && n_ok)
+                           ? bf16_to_f32(e.residual[static_cast<int64_t>(m) * e.n_out + n])
+                           : 0.0f;
+            }
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const int m = mbase + j;
+                const float z = __uint_as_float(v[j]) + b;
+                const float h = (e.act == kActGELU ? gelu_f32(z) : z) + r[j];
+                if (m < p.M && n_ok) p.out[static_cast<int64_t>(m) * e.n_out + n] = f32_to_bf16_rn(h);
+            }
+        }
+    }
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int MIN_BLOCKS>
-__global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
+// Plain epilogue of one tile: bf16 stores of the accumulators; for even N
+// neighbouring lanes pair up so that each store writes two adjacent outputs
+// (n, n+1) of one token as a 32-bit word.
+template <int T>
+__device__ __forceinline__ void plain_epilogue_tile(const TsParams& p, uint32_t d_col, int m0,
+                                                    int n, int lane, bool n_even, int c0, int cs) {
+#pragma unroll 1
+    for (int c = c0; c < T / 32; c += cs) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(d_col + c * 32, v);
+        tmem_ld_wait(v);
+        const int mbase = m0 + c * 32;
+        if (n_even) {
+            // Pair neighbouring lanes so that each store writes two
+            // adjacent outputs (n, n+1) of one token as a 32-bit word.
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float f0 = __uint_as_float(v[2 * j]);
+                const float f1 = __uint_as_float(v[2 * j + 1]);
+                const float send = (lane & 1) ? f0 : f1;
+                const float other = __shfl_xor_sync(0xffffffffu, send, 1);
+                int m, col;
+                uint32_t word;
+                if ((lane & 1) == 0) {
+                    m = mbase + 2 * j;
+                    col = n;
+                    word = pack_bf16x2(f0, other);
+                } else {
+                    m = mbase + 2 * j + 1;
+                    col = n - 1;
+                    word = pack_bf16x2(other, f1);
+                }
+                if (m < p.M && col < p.N)
+                    *reinterpret_cast<uint32_t*>(p.out + static_cast<int64_t>(m) * p.N +
+                                                 col) = word;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const int m = mbase + j;
+                if (m < p.M && n < p.N) {
+                    const uint32_t word = pack_bf16x2(__uint_as_float(v[j]), 0.0f);
+                    p.out[static_cast<int64_t>(m) * p.N + n] =
+                        static_cast<uint16_t>(word & 0xFFFFu);
+                }
+            }
+        }
+    }
+}
+
+template <int DQ, int EP>
+constexpr int threads_for() {
+    return 32 * (2 + 4 * DQ + 4 * EP);
+}
+
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED>
+__global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
     using L = Layout<T, S_SMEM, S_TMEM>;
@@ -124,7 +268,7 @@ __global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
             mbar_init(empty_a(s), 1);
         }
         mbar_init(d_full, 1);
-        mbar_init(d_empty, 4);  // one arrival per epilogue warp
+        mbar_init(d_empty, 4 * EP);  // one arrival per epilogue warp
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -288,7 +432,9 @@ __global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
         }
     } else {
         // ------------------------------------------------------------ epilogue
+        // EP groups of four warps; group eg takes the 32-token chunks eg, eg + EP, ...
         const int sub = warp & 3;
+        const int eg = (warp - (2 + 4 * DQ)) >> 2;
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const bool n_even = (p.N & 1) == 0;
         uint32_t tcount = 0;
@@ -299,48 +445,10 @@ __global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
                 break;
             tc_fence_after();
             const int n = wt * kRows + sub * 32 + lane;
-#pragma unroll 1
-            for (int c = 0; c < T / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(lane_base + L::D_COL + c * 32, v);
-                tmem_ld_wait(v);
-                const int mbase = tt * T + c * 32;
-                if (n_even) {
-                    // Pair neighbouring lanes so that each store writes two
-                    // adjacent outputs (n, n+1) of one token as a 32-bit word.
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const float f0 = __uint_as_float(v[2 * j]);
-                        const float f1 = __uint_as_float(v[2 * j + 1]);
-                        const float send = (lane & 1) ? f0 : f1;
-                        const float other = __shfl_xor_sync(0xffffffffu, send, 1);
-                        int m, col;
-                        uint32_t word;
-                        if ((lane & 1) == 0) {
-                            m = mbase + 2 * j;
-                            col = n;
-                            word = pack_bf16x2(f0, other);
-                        } else {
-                            m = mbase + 2 * j + 1;
-                            col = n - 1;
-                            word = pack_bf16x2(other, f1);
-                        }
-                        if (m < p.M && col < p.N)
-                            *reinterpret_cast<uint32_t*>(p.out + static_cast<int64_t>(m) * p.N +
-                                                         col) = word;
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int m = mbase + j;
-                        if (m < p.M && n < p.N) {
-                            const uint32_t word = pack_bf16x2(__uint_as_float(v[j]), 0.0f);
-                            p.out[static_cast<int64_t>(m) * p.N + n] =
-                                static_cast<uint16_t>(word & 0xFFFFu);
-                        }
-                    }
-                }
-            }
+            if constexpr (FUSED)
+                fused_epilogue_tile<T>(p, lane_base + L::D_COL, tt * T, n, lane, eg, EP);
+            else
+                plain_epilogue_tile<T>(p, lane_base + L::D_COL, tt * T, n, lane, n_even, eg, EP);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(d_empty);
@@ -353,16 +461,20 @@ __global__ void __launch_bounds__(threads_for<DQ>(), MIN_BLOCKS)
     if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int MIN_BLOCKS>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS>
 cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
                            int grid, cudaStream_t stream) {
     using L = Layout<T, S_SMEM, S_TMEM>;
-    auto kern = w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, MIN_BLOCKS>;
+    // the plain variant carries none of the fused epilogue's code or registers
+    const bool fused =
+        p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
+    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true>
+                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false>;
     // Idempotent; cheap enough to repeat per launch and per device.
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    kern<<<grid, threads_for<DQ>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    kern<<<grid, threads_for<DQ, EP>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
     return cudaGetLastError();
 }
 
@@ -374,10 +486,14 @@ cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const T
 #ifndef W4A16_GEMM_SS
 #define W4A16_GEMM_SS 6
 #endif
-constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ;
+#ifndef W4A16_GEMM_EP
+#define W4A16_GEMM_EP 2
+#endif
+constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ,
+              kGemmEP = W4A16_GEMM_EP;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
-constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1;
+constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
 
 }  // namespace
 
@@ -391,8 +507,9 @@ int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
                       const TsParams& p, int grid, cudaStream_t stream) {
     if (v == TsVariant::kGemm256)
-        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, 1>(tx, tw, p, grid, stream);
-    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, 3>(tx, tw, p, grid, stream);
+        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1>(tx, tw, p, grid,
+                                                                            stream);
+    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3>(tx, tw, p, grid, stream);
 }
 
 }  // namespace w4a16

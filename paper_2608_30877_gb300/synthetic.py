@@ -48,6 +48,9 @@ TINY = LinearCase("tiny_64x512x1024", 64, 1024, 512, GROUP, 0, 0)
 QKV_PREFILL = LinearCase("qkv_prefill_4096x12288x36864", 4096, 3 * D_MODEL, D_MODEL, GROUP, 1, 1)
 MLP_UP = LinearCase("mlp_up_8192x12288x49152", 8192, D_FF, D_MODEL, GROUP, 2, 2)
 MLP_DOWN = LinearCase("mlp_down_8192x49152x12288", 8192, D_MODEL, D_FF, GROUP, 2, 3)
+# gate and up projections as one matrix of interleaved rows (gate 2j, up 2j+1),
+# run with the fused SwiGLU epilogue: [8192, 12288] -> [8192, 49152]
+MLP_SWIGLU = LinearCase("mlp_swiglu_8192x12288x2x49152", 8192, 2 * D_FF, D_MODEL, GROUP, 2, 4)
 GEMV_MS = (1, 8, 16, 32)
 
 

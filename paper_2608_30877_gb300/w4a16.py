@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libw4a16.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "w4a16.h")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_ALIGNMENT, ERR_CUDA, ERR_TIMEOUT = range(6)
+ACT_NONE, ACT_SWIGLU, ACT_GELU = range(3)
 
 _lib = None
 
@@ -49,6 +50,7 @@ def lib() -> ctypes.CDLL:
         L = ctypes.CDLL(LIB_PATH)
         i64, p = ctypes.c_int64, ctypes.c_void_p
         L.w4a16_linear.argtypes = [p, p, p, p, i64, i64, i64, i64, p]
+        L.w4a16_linear_fused.argtypes = [p, p, p, p, p, p, i64, i64, i64, i64, ctypes.c_int, p]
         L.w4a16_linear_stack.argtypes = [ctypes.POINTER(Layer), i64, i64, i64, p]
         L.w4a16_dequant.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_quantize.argtypes = [p, p, p, i64, i64, i64, p]
@@ -57,7 +59,7 @@ def lib() -> ctypes.CDLL:
         L.w4a16_status_string.argtypes = [ctypes.c_int]
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
-        for f in ("w4a16_linear", "w4a16_linear_stack", "w4a16_dequant", "w4a16_quantize",
+        for f in ("w4a16_linear", "w4a16_linear_fused", "w4a16_linear_stack", "w4a16_dequant", "w4a16_quantize",
                   "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
@@ -102,6 +104,26 @@ def linear(x: torch.Tensor, w_packed: torch.Tensor, scales: torch.Tensor, g: int
     assert w_packed.shape[1] * 2 == K and scales.shape == (N, K // g) and out.shape == (M, N)
     _check("w4a16_linear", lib().w4a16_linear(x.data_ptr(), w_packed.data_ptr(), scales.data_ptr(),
                                               out.data_ptr(), M, N, K, g, _stream(stream)))
+    return out
+
+
+def linear_fused(x: torch.Tensor, w_packed: torch.Tensor, scales: torch.Tensor, g: int = 128,
+                 act: int = ACT_NONE, bias: torch.Tensor | None = None,
+                 residual: torch.Tensor | None = None, out: torch.Tensor | None = None,
+                 stream=None) -> torch.Tensor:
+    """out = act(x @ dequant(w)^T + bias) + residual (include/w4a16.h); for
+    ACT_SWIGLU rows (2j, 2j+1) of w are (gate, up) and out has N/2 columns."""
+    M, K = x.shape
+    N = w_packed.shape[0]
+    n_out = N // 2 if act == ACT_SWIGLU else N
+    if out is None:
+        out = torch.empty((M, n_out), dtype=torch.bfloat16, device=x.device)
+    _need_cuda(x, w_packed, scales, out, *(t for t in (bias, residual) if t is not None))
+    _check("w4a16_linear_fused", lib().w4a16_linear_fused(
+        x.data_ptr(), w_packed.data_ptr(), scales.data_ptr(),
+        None if bias is None else bias.data_ptr(),
+        None if residual is None else residual.data_ptr(),
+        out.data_ptr(), M, N, K, g, int(act), _stream(stream)))
     return out
 
 

@@ -40,3 +40,37 @@ def assert_close(gpu: np.ndarray, ref: np.ndarray, what: str = ""):
     assert m["max_err_over_rms"] <= MAX_ERR_OVER_RMS, f"{what}: {m}"
     assert m["rel_fro"] <= REL_FRO, f"{what}: {m}"
     return m
+
+
+def assert_close_fused(gpu: np.ndarray, y: np.ndarray, ref: np.ndarray, act: int,
+                       bias=None, what: str = ""):
+    """Tolerance for fused-epilogue outputs h = act(y + bias) + residual.
+
+    The plain-linear bound allows the pre-activation y an error of up to
+    MAX_ERR_OVER_RMS * rms(y) per element (fp32 accumulation in any order, and
+    in the small-M kernel the scale applied per group in fp32 instead of a
+    bf16 rounding of every (q - 8) s).  The activation carries that error
+    scaled by its derivative: 1 (none), |GELU'(z)|, and for SwiGLU
+    |silu'(g) u| + |silu(g)| (gate g, up u).  On top comes the bf16 store,
+    half an ulp, i.e. at most 2^-9 |ref|; the bound takes twice each term.
+    The Frobenius bound is the plain one."""
+    from math import sqrt
+    y = np.asarray(y, dtype=np.float64)
+    z = y + (0.0 if bias is None else O.bf16_bits_to_f32(np.asarray(bias)).astype(np.float64))
+    eps = 2.0 * MAX_ERR_OVER_RMS * float(np.sqrt(np.mean(y * y)))
+    if act == 1:
+        gate, up = z[:, 0::2], z[:, 1::2]
+        sig = 1.0 / (1.0 + np.exp(-gate))
+        gain = np.abs(sig * (1.0 + gate * (1.0 - sig)) * up) + np.abs(gate * sig)
+    elif act == 2:
+        from scipy.special import erf
+        gain = np.abs(0.5 * (1.0 + erf(z / sqrt(2.0))) + z * np.exp(-0.5 * z * z) / sqrt(2.0 * np.pi))
+    else:
+        gain = np.ones_like(z)
+    m = O.error_metrics(gpu, ref)
+    assert np.isfinite(gpu).all(), f"{what}: non-finite output"
+    bound = 2.0 ** -8 * np.abs(ref) + eps * gain + 1e-30
+    worst = float(np.max(np.abs(gpu - ref) / bound)) if ref.size else 0.0
+    assert worst <= 1.0, f"{what}: worst error / bound = {worst:.3f}, {m}"
+    assert m["rel_fro"] <= REL_FRO, f"{what}: {m}"
+    return m

@@ -66,3 +66,17 @@ def test_dequant_and_quantize_reject_bad_args(L):
     assert L.w4a16_dequant(A, 2 * A, 3 * A + 4, 8, 256, 128, None) == W.ERR_ALIGNMENT
     assert L.w4a16_quantize(0, 2 * A, 3 * A, 8, 256, 128, None) == W.ERR_INVALID_ARG
     assert L.w4a16_quantize(A, 2 * A, 3 * A, 8, 256, 48, None) == W.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("bias,res,out,N,act,want", [
+    (0, 0, 4 * A, 8, 3, W.ERR_INVALID_ARG),             # unknown activation
+    (0, 0, 4 * A, 7, W.ACT_SWIGLU, W.ERR_INVALID_ARG),  # SwiGLU needs even N
+    (5 * A + 2, 0, 4 * A, 8, W.ACT_GELU, W.ERR_ALIGNMENT),   # misaligned bias
+    (0, 6 * A + 8, 4 * A, 8, W.ACT_NONE, W.ERR_ALIGNMENT),   # misaligned residual
+    (4 * A + 16, 0, 4 * A, 8, W.ACT_NONE, W.ERR_INVALID_ARG),  # bias overlaps out
+    (0, 4 * A + 16, 4 * A, 8, W.ACT_NONE, W.ERR_INVALID_ARG),  # residual partly overlaps out
+    (0, 0, A + 64, 8, W.ACT_SWIGLU, W.ERR_INVALID_ARG),        # out overlaps x
+])
+def test_fused_rejects_before_launch(L, bias, res, out, N, act, want):
+    assert L.w4a16_linear_fused(A, 2 * A, 3 * A, bias or None, res or None, out, 4, N, 256, 128,
+                                act, None) == want
