@@ -57,6 +57,9 @@ def lib():
         L.oracle_linear_rows.argtypes = [p, p, p, i64, i64, i64, i64, p, i64, p, ctypes.c_int]
         L.oracle_linear_points.argtypes = [p, p, p, i64, i64, i64, i64, p, p, i64, p, ctypes.c_int]
         L.oracle_epilogue_rows.argtypes = [p, i64, i64, p, p, p, ctypes.c_int, p]
+        L.oracle_gather_rows.argtypes = [p, i64, i64, p, i64, p]
+        L.oracle_gather_rows.restype = ctypes.c_int
+        L.oracle_topk_smallest.argtypes = [p, i64, i64, p, p, p]
         L.oracle_max_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -167,6 +170,29 @@ def epilogue_rows(y: np.ndarray, act: int = ACT_NONE, bias=None, residual=None,
     lib().oracle_epilogue_rows(_ptr(y), nrows, N, None if b is None else _ptr(b),
                                None if res is None else _ptr(res), _ptr(rows), int(act), _ptr(out))
     return out
+
+
+def gather_rows(src_bits: np.ndarray, idx) -> tuple[np.ndarray, bool]:
+    """dst[p] = src[idx[p]] (bf16 bits); out-of-range indices give zero rows
+    and ok = False."""
+    src_bits = np.ascontiguousarray(src_bits, dtype=np.uint16)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    rows, D = src_bits.shape
+    dst = np.empty((idx.shape[0], D), dtype=np.uint16)
+    bad = lib().oracle_gather_rows(_ptr(src_bits), rows, D, _ptr(idx), idx.shape[0], _ptr(dst))
+    return dst, bad == 0
+
+
+def topk_smallest(scores: np.ndarray, k: int):
+    """(indices int32 [k], scores fp32 [k]) of the k smallest scores, ascending
+    by IEEE totalOrder (NaN last), ties by index."""
+    scores = np.ascontiguousarray(scores, dtype=np.float32)
+    n = scores.shape[0]
+    idx = np.empty(k, dtype=np.int32)
+    val = np.empty(k, dtype=np.float32)
+    taken = np.empty(max(n, 1), dtype=np.uint8)
+    lib().oracle_topk_smallest(_ptr(scores), n, k, _ptr(idx), _ptr(val), _ptr(taken))
+    return idx, val
 
 
 def max_threads() -> int:

@@ -225,6 +225,64 @@ void oracle_epilogue_rows(const double* y, int64_t nrows, int64_t N, const uint1
     }
 }
 
+/* ---- scoring readout: gather and top-k ------------------------------------
+ *
+ * The pipeline's last modules (Sec. 3.3): the affinity head reads one hidden
+ * state per pair (rows of the packed batch picked by index), and the
+ * predicted affinities are sorted for export.  Readings fixed for this
+ * library: affinities are binding free energies in kcal/mol, so the best
+ * candidates are the k smallest; scores are ordered by the IEEE 754
+ * totalOrder predicate on non-NaN values (-0 before +0), every NaN after
+ * every number, and equal scores by ascending index. */
+
+/* dst[p, :] = src[idx[p], :]; an index outside [0, src_rows) gives a zero row
+ * and a nonzero return. */
+int oracle_gather_rows(const uint16_t* src, int64_t src_rows, int64_t D, const int32_t* idx,
+                       int64_t P, uint16_t* dst) {
+    int bad = 0;
+    for (int64_t p = 0; p < P; ++p) {
+        if (idx[p] < 0 || idx[p] >= src_rows) {
+            for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 0;
+            bad = 1;
+            continue;
+        }
+        for (int64_t d = 0; d < D; ++d) dst[p * D + d] = src[(int64_t)idx[p] * D + d];
+    }
+    return bad;
+}
+
+/* -1, 0, 1 as (a, ia) orders before, equal to, after (b, ib). */
+static int score_order(float a, int64_t ia, float b, int64_t ib) {
+    int na = isnan(a) != 0, nb = isnan(b) != 0;
+    if (na != nb) return na ? 1 : -1;          /* NaN after every number */
+    if (!na) {
+        if (a < b) return -1;
+        if (a > b) return 1;
+        if (a == 0.0f) {                        /* equal zeros: -0 before +0 */
+            int sa = signbit(a) != 0, sb = signbit(b) != 0;
+            if (sa != sb) return sa ? -1 : 1;
+        }
+    }
+    return ia < ib ? -1 : (ia > ib ? 1 : 0);   /* ties by index */
+}
+
+/* The k smallest scores in order: out_idx[j], out_val[j] for j < k, by
+ * repeated selection of the least remaining element (O(n k), plain). */
+void oracle_topk_smallest(const float* scores, int64_t n, int64_t k, int32_t* out_idx,
+                          float* out_val, unsigned char* taken) {
+    memset(taken, 0, (size_t)n);
+    for (int64_t j = 0; j < k; ++j) {
+        int64_t best = -1;
+        for (int64_t i = 0; i < n; ++i) {
+            if (taken[i]) continue;
+            if (best < 0 || score_order(scores[i], i, scores[best], best) < 0) best = i;
+        }
+        taken[best] = 1;
+        out_idx[j] = (int32_t)best;
+        out_val[j] = scores[best];
+    }
+}
+
 int oracle_max_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

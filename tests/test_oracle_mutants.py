@@ -4,7 +4,9 @@ Each case compiles a copy of oracle/w4a16_oracle.c with one planted mistake
 (swapped nibbles, dropped zero point, wrong group index, round-half-away,
 truncating bf16 rounding, fp32 accumulation, wrong activation row, and in
 the fused epilogue swapped gate/up, a wrong SiLU sign, the tanh GELU
-approximation, a wrong residual row, bias after the activation), points
+approximation, a wrong residual row, bias after the activation; in the
+readout top-k ties by the last index, unordered zeros, NaN first, and a gather
+that does not zero the rows of bad indices), points
 the oracle module at it and runs the pins: at least one must fail.  The
 mistakes live only in temporary copies on the CPU."""
 import ctypes
@@ -34,6 +36,12 @@ MUTANTS = {
     "residual_wrong_row": [("residual[rows[r] * n_out + j]", "residual[r * n_out + j]")],
     "bias_after_activation": [("h = act == 2 ? gelu_d(z) : z;",
                                "h = act == 2 ? gelu_d(yr[j]) + (z - yr[j]) : z;")],
+    "topk_ties_by_last_index": [("return ia < ib ? -1 : (ia > ib ? 1 : 0);",
+                                 "return ia > ib ? -1 : (ia < ib ? 1 : 0);")],
+    "topk_zeros_unordered": [("if (sa != sb) return sa ? -1 : 1;", "(void)sa; (void)sb;")],
+    "topk_nan_first": [("if (na != nb) return na ? 1 : -1;", "if (na != nb) return na ? -1 : 1;")],
+    "gather_bad_rows_not_zeroed": [("for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 0;",
+                                    "for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 1;")],
 }
 
 PINS = [
@@ -54,6 +62,9 @@ PINS = [
     P.test_epilogue_gelu_normal_cdf_values,
     P.test_epilogue_bias_residual_by_hand,
     P.test_epilogue_bias_enters_before_the_activation,
+    P.test_gather_rows_by_hand,
+    P.test_topk_hand_example_ties_zeros_nan,
+    P.test_topk_matches_a_textbook_sort,
 ]
 
 
@@ -78,7 +89,8 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
         mut = ctypes.CDLL(so)
         for fn in ("oracle_bf16_rne", "oracle_bf16_to_f32", "oracle_unpack", "oracle_pack",
                    "oracle_quantize", "oracle_dequant", "oracle_linear_rows",
-                   "oracle_linear_points", "oracle_epilogue_rows", "oracle_max_threads"):
+                   "oracle_linear_points", "oracle_epilogue_rows", "oracle_gather_rows",
+                   "oracle_topk_smallest", "oracle_max_threads"):
             getattr(mut, fn).argtypes = getattr(good, fn).argtypes
             getattr(mut, fn).restype = getattr(good, fn).restype
         monkeypatch.setattr(O, "_lib", mut)

@@ -349,3 +349,40 @@ def test_epilogue_bias_enters_before_the_activation():
     assert abs(h[0, 0] - 3.0 * math.e / (1.0 + math.e)) < 1e-15
     hg = O.epilogue_rows(np.array([[0.0]]), O.ACT_GELU, bias=np.array([0x3F80], dtype=np.uint16))
     assert abs(hg[0, 0] - 0.8413447460685429) < 1e-15
+
+
+# ---- scoring readout: gather and top-k (Sec. 3.3: affinity prediction, then
+# result sorting; the best binders have the smallest free energy) -----------
+
+def test_gather_rows_by_hand():
+    src = np.arange(12, dtype=np.uint16).reshape(4, 3)
+    dst, ok = O.gather_rows(src, [3, 0, 3])
+    assert ok and dst.tolist() == [[9, 10, 11], [0, 1, 2], [9, 10, 11]]
+    dst, ok = O.gather_rows(src, [1, 4, -1])
+    assert not ok and dst.tolist() == [[3, 4, 5], [0, 0, 0], [0, 0, 0]]
+
+
+def test_topk_hand_example_ties_zeros_nan():
+    s = np.array([3.0, -1.0, np.nan, -1.0, 0.0, -0.0, 2.5], dtype=np.float32)
+    idx, val = O.topk_smallest(s, 7)
+    assert idx.tolist() == [1, 3, 5, 4, 6, 0, 2]       # -1 (idx 1, 3), -0, +0, 2.5, 3, NaN
+    assert np.signbit(val[2]) and not np.signbit(val[3])
+    idx, _ = O.topk_smallest(s, 2)
+    assert idx.tolist() == [1, 3]
+    idx, _ = O.topk_smallest(np.array([np.nan, np.nan, 5.0], dtype=np.float32), 3)
+    assert idx.tolist() == [2, 0, 1]                    # NaNs last, by index
+
+
+def test_topk_matches_a_textbook_sort():
+    # totalOrder on non-NaN floats with ties by index = a stable sort of the
+    # (value, -0 before +0) keys; check against Python's sorted on random data
+    rng = np.random.default_rng(11)
+    s = rng.normal(size=500).astype(np.float32)
+    s[rng.integers(0, 500, 40)] = 0.25                  # many ties
+    s[rng.integers(0, 500, 5)] = -0.0
+    s[rng.integers(0, 500, 5)] = 0.0
+    order = sorted(range(500), key=lambda i: (float(s[i]), 0 if np.signbit(s[i]) else 1, i))
+    for k in (1, 17, 500):
+        idx, val = O.topk_smallest(s, k)
+        assert idx.tolist() == order[:k]
+        assert val.tobytes() == s[order[:k]].tobytes()
