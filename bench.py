@@ -43,7 +43,7 @@ NCU_TRAFFIC = {
     # QKV prefill 4096x12288x36864, one launch (full capture)
     ("qkv", "ts", "cf808ae786339c73"): 1.175e9 + 0.295e9,
     # small-M readout, M = 8, 12288x49152 (full capture)
-    ("gemv", "gemv", "86533d1fc49622b2"): 0.3186e9 + 0.0038e9,
+    ("gemv", "gemv", "cfa826941725038f"): 0.3188e9 + 0.0036e9,
 }
 
 KERNEL_FILES = {"ts": ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"),
@@ -60,6 +60,8 @@ def kernel_source_hash(kind: str = "ts") -> str:
 
 
 def ncu_traffic(config: str, m: int):
+    if config == "topk":
+        return None  # no capture of the readout kernels is summarised
     if config == "gemv":
         if m > 8:  # the capture is of the M <= 8 instantiation
             return None
@@ -278,6 +280,26 @@ class LinearWorkload:
             W.linear(self.x, packed, scales, self.g, out=self.out, stream=stream)
 
 
+class TopkWorkload:
+    """Result sorting of the screening set: the k best (smallest) of n
+    predicted affinities, fp32 scores resident on the device."""
+
+    def __init__(self, n, k, seed):
+        import torch
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed)
+        self.name, self.n, self.k = f"topk_n{n}_k{k}", n, k
+        self.x = torch.randn(n, generator=g, device="cuda") * 2.0 - 8.0   # kcal/mol-like
+        self.out = torch.empty(k, dtype=torch.float32, device="cuda")
+        self.flops = 0.0
+        self.bytes = 4.0 * n + 8.0 * k       # scores read once, (index, score) written once
+        self.launches_per_step = 1
+
+    def step(self, stream=None):
+        from paper_2608_30877_gb300 import w4a16 as W
+        _, self.out = W.topk_smallest(self.x, self.k, stream=stream)
+
+
 # ----------------------------------------------------------------- CPU oracle
 
 def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 2048):
@@ -305,6 +327,23 @@ def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 2048):
         r = min(rows_max, max(r + 1, int(r * (target_s / 2) / max(dt, 1e-3))))
 
 
+def oracle_topk_sample(n: int, k: int):
+    """Times the oracle's top-k (plain repeated selection, one thread) on the
+    same n seeded scores with k reduced to fit ~10 s; returns (GB/s of the
+    algorithmic bytes 4 n + 8 k scaled to the full k, description)."""
+    import numpy as np
+    from oracle import oracle as O
+    s = (np.random.default_rng(5).normal(size=n) * 2.0 - 8.0).astype(np.float32)
+    kk = max(1, min(k, 50))
+    t0 = time.perf_counter()
+    O.topk_smallest(s, kk)
+    dt = time.perf_counter() - t0
+    t_full = dt * k / kk                  # selection time grows linearly in k
+    desc = (f"oracle top-k by repeated selection, n={n}, k={kk} in {dt:.2f} s on 1 thread, "
+            f"scaled linearly to k={k}")
+    return (4.0 * n + 8.0 * k) / t_full / 1e9, desc
+
+
 def stack_macs_per_pair(tokens=1024, layers=96):
     from paper_2608_30877_gb300 import synthetic as S
     return tokens * layers * sum(N * K for (_, K, N) in S.LAYER_LINEARS)
@@ -322,6 +361,10 @@ def config_for(args):
                 "pairs": args.pairs, "tokens_per_pair": 1024, "layers": args.layers, "g": 128,
                 "l2": "inputs larger than L2 (88 GB packed weights, >=1.6 GB activations per "
                       "linear); no flush"}
+    if c == "topk":
+        return {"workload": f"top-k of predicted affinities, n={args.topk_n}, k={args.topk_k}",
+                "n": args.topk_n, "k": args.topk_k,
+                "l2": "scores (<1 MB) stay in L2: the step is latency-bound; no flush"}
     cases = {"qkv": S.QKV_PREFILL, "mlp_up": S.MLP_UP, "mlp_down": S.MLP_DOWN, "tiny": S.TINY,
              "mlp_swiglu": S.MLP_SWIGLU}
     if c == "gemv":
@@ -341,6 +384,24 @@ def run_reference(args):
     if rank != 0:
         return 0
     from paper_2608_30877_gb300 import synthetic as S
+    if args.config == "topk":
+        vals, desc = [], ""
+        for i in range(args.warmup + args.steps):
+            gbs, desc = oracle_topk_sample(args.topk_n, args.topk_k)
+            if i >= args.warmup:
+                vals.append(gbs)
+        value = statistics.median(vals)
+        line = {"metric": METRIC, "impl": "reference", "value": value, "unit": "GB/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": 1e3 * (4.0 * args.topk_n + 8.0 * args.topk_k) / value / 1e9,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic", "config": config_for(args),
+                "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                 "sample": desc},
+                "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
     if args.config == "stack":
         K, N_rows = S.D_MODEL, 2048
         unit = "pairs/s"
@@ -377,7 +438,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="stack",
-                    choices=["stack", "qkv", "mlp_up", "mlp_down", "mlp_swiglu", "gemv", "tiny"])
+                    choices=["stack", "qkv", "mlp_up", "mlp_down", "mlp_swiglu", "gemv", "tiny",
+                             "topk"])
+    ap.add_argument("--topk-n", type=int, default=200000, help="scores for --config topk")
+    ap.add_argument("--topk-k", type=int, default=1000, help="k for --config topk")
     ap.add_argument("--m", type=int, default=32, help="tokens for --config gemv")
     ap.add_argument("--pairs", type=int, default=64)
     ap.add_argument("--layers", type=int, default=96)
@@ -403,6 +467,10 @@ def main():
         wl = StackWorkload(args.pairs, 1024, args.layers)
         unit = "pairs/s"
         units_per_step = wl.pairs
+    elif args.config == "topk":
+        wl = TopkWorkload(args.topk_n, args.topk_k, 5)
+        unit = "GB/s"
+        units_per_step = None
     else:
         from paper_2608_30877_gb300 import synthetic as S
         cfg = config_for(args)
@@ -436,14 +504,14 @@ def main():
 
     if args.config == "stack":
         value = world * units_per_step / step_s
-    elif args.config == "gemv":
+    elif args.config in ("gemv", "topk"):
         value = world * wl.bytes / step_s / 1e9
     else:
         value = world * wl.flops / step_s / 1e12
 
     # roofline of the fused kernel: every launch in the step is that kernel
     per_launch_s = step_s / wl.launches_per_step
-    if args.config == "gemv":
+    if args.config in ("gemv", "topk"):
         achieved = wl.bytes / step_s / 1e9
         peak = peaks["hbm_gbs"]
         roof = {"bound": "hbm", "unit": "GB/s"}
@@ -455,7 +523,7 @@ def main():
     roof.update({"achieved": achieved, "peak": peak, "frac": achieved / peak,
                  "traffic": traffic, "peak_source": peaks["source"] + (
                      " bf16_tflops_sustained" if args.config == "stack" else
-                     (" hbm_gbs" if args.config == "gemv" else " bf16_tflops")),
+                     (" hbm_gbs" if args.config in ("gemv", "topk") else " bf16_tflops")),
                  "per_launch_ms": per_launch_s * 1e3,
                  "algorithmic_bytes_per_step": wl.bytes, "flops_per_step": wl.flops})
 
@@ -475,7 +543,11 @@ def main():
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         from paper_2608_30877_gb300 import synthetic as S
-        if args.config == "stack":
+        if args.config == "topk":
+            gbs, desc = oracle_topk_sample(args.topk_n, args.topk_k)
+            line["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                    "sample": desc}
+        elif args.config == "stack":
             mac_s, desc, threads = oracle_sample(S.D_MODEL, 2048, 15.0)
             cb = mac_s / stack_macs_per_pair(1024, args.layers)
             line["cpu_baseline"] = {"value": cb, "unit": "pairs/s", "cores": threads,

@@ -153,6 +153,39 @@ int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales_bf16,
                    int64_t N, int64_t K, int64_t g, void* stream);
 
 /*
+ * Scoring readout, the last modules of the screening pipeline (Sec. 3.3):
+ * the affinity head reads one hidden state per pair of the packed batch
+ * (w4a16_gather_rows, then w4a16_linear_fused with the head's weights and
+ * bias), and the predicted affinities are sorted for export
+ * (w4a16_topk_smallest).
+ *
+ * dst_bf16[p, :] = src_bf16[index_i32[p], :] for p < P.
+ *   src_bf16   [src_rows, D] bf16, device
+ *   index_i32  [P] int32, device (e.g. the last token of each pair)
+ *   dst_bf16   [P, D] bf16, device, must not overlap src or the index
+ * An index outside [0, src_rows) gives a zero row and records
+ * W4A16_ERR_INVALID_ARG in the device status word (w4a16_get_device_error).
+ */
+int w4a16_gather_rows(const void* src_bf16, int64_t src_rows, int64_t D,
+                      const void* index_i32, int64_t P, void* dst_bf16, void* stream);
+
+/*
+ * The k smallest of n scores -- predicted binding free energies in kcal/mol,
+ * so the best binders -- in ascending order: out_index_i32[j] is the index
+ * and out_score_f32[j] the score of the j-th.  Order: IEEE 754 totalOrder on
+ * numbers (-0 before +0), every NaN after every number, equal scores by
+ * ascending index; the result is unique and deterministic.
+ *   scores         [n] device, fp32 (score_bits = 32) or bf16 (score_bits =
+ *                  16, e.g. the head's output; widened exactly to fp32),
+ *                  1 <= n < 2^31; other score_bits: W4A16_ERR_INVALID_ARG
+ *   1 <= k <= n, k <= 1024 (larger k: W4A16_ERR_UNSUPPORTED)
+ *   out_index_i32  [k] int32, out_score_f32 [k] fp32, device, disjoint
+ * One launch of one 8-CTA thread-block cluster; no scratch memory.
+ */
+int w4a16_topk_smallest(const void* scores, int score_bits, int64_t n, int64_t k,
+                        void* out_index_i32, void* out_score_f32, void* stream);
+
+/*
  * Synchronises `stream`, then reads and clears the device status word that
  * kernels set when a bounded wait runs out.  Returns W4A16_OK,
  * W4A16_ERR_TIMEOUT or W4A16_ERR_CUDA.

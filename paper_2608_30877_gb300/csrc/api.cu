@@ -333,6 +333,54 @@ extern "C" int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales
                : W4A16_ERR_CUDA;
 }
 
+extern "C" int w4a16_gather_rows(const void* src_bf16, int64_t src_rows, int64_t D,
+                                 const void* index_i32, int64_t P, void* dst_bf16,
+                                 void* stream) {
+    if (src_bf16 == nullptr || index_i32 == nullptr || dst_bf16 == nullptr)
+        return W4A16_ERR_INVALID_ARG;
+    if (src_rows <= 0 || D <= 0 || P <= 0) return W4A16_ERR_INVALID_ARG;
+    if (src_rows > kMaxDim || D > kMaxDim || P > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(src_bf16) || !aligned16(index_i32) || !aligned16(dst_bf16))
+        return W4A16_ERR_ALIGNMENT;
+    if (overlaps(dst_bf16, P * D * 2, src_bf16, src_rows * D * 2) ||
+        overlaps(dst_bf16, P * D * 2, index_i32, P * 4))
+        return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    const int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    return launch_gather_rows(static_cast<const uint16_t*>(src_bf16), src_rows, D,
+                              static_cast<const int32_t*>(index_i32), P,
+                              static_cast<uint16_t*>(dst_bf16), st->status, st->sm_count,
+                              static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_topk_smallest(const void* scores, int score_bits, int64_t n, int64_t k,
+                                   void* out_index_i32, void* out_score_f32, void* stream) {
+    if (scores == nullptr || out_index_i32 == nullptr || out_score_f32 == nullptr)
+        return W4A16_ERR_INVALID_ARG;
+    if (score_bits != 32 && score_bits != 16) return W4A16_ERR_INVALID_ARG;
+    if (n <= 0 || k <= 0 || k > n) return W4A16_ERR_INVALID_ARG;
+    if (k > kTopkMaxK || n > kMaxDim) return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(scores) || !aligned16(out_index_i32) || !aligned16(out_score_f32))
+        return W4A16_ERR_ALIGNMENT;
+    const int64_t in_bytes = n * (score_bits / 8);
+    if (overlaps(out_index_i32, k * 4, scores, in_bytes) ||
+        overlaps(out_score_f32, k * 4, scores, in_bytes) ||
+        overlaps(out_index_i32, k * 4, out_score_f32, k * 4))
+        return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    const int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    return launch_topk_smallest(scores, score_bits == 16, n, static_cast<int>(k),
+                                static_cast<int32_t*>(out_index_i32),
+                                static_cast<float*>(out_score_f32),
+                                static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
 extern "C" int w4a16_get_device_error(void* stream) {
     DeviceState* st = nullptr;
     int rc = device_state(&st);

@@ -63,6 +63,14 @@ int gemv_tokens_per_tile(int64_t M);
 cudaError_t gemv_launch(const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                         const GemvParams& p, int sm_count, cudaStream_t stream);
 
+// Scoring readout (readout.cu).
+constexpr int kTopkMaxK = 1024;  // largest k of the top-k
+cudaError_t launch_topk_smallest(const void* scores, bool bf16, int64_t n, int k,
+                                 int32_t* out_idx, float* out_val, cudaStream_t stream);
+cudaError_t launch_gather_rows(const uint16_t* src, int64_t src_rows, int64_t D,
+                               const int32_t* idx, int64_t P, uint16_t* dst, int* status,
+                               int sm_count, cudaStream_t stream);
+
 cudaError_t launch_dequant(const uint8_t* w, const uint16_t* scales, uint16_t* wd, int64_t N,
                            int64_t K, int64_t g, cudaStream_t stream);
 cudaError_t launch_quantize(const float* w, uint8_t* packed, uint16_t* scales, int64_t N,

@@ -53,13 +53,16 @@ def lib() -> ctypes.CDLL:
         L.w4a16_linear_fused.argtypes = [p, p, p, p, p, p, i64, i64, i64, i64, ctypes.c_int, p]
         L.w4a16_linear_stack.argtypes = [ctypes.POINTER(Layer), i64, i64, i64, p]
         L.w4a16_dequant.argtypes = [p, p, p, i64, i64, i64, p]
+        L.w4a16_gather_rows.argtypes = [p, i64, i64, p, i64, p, p]
+        L.w4a16_topk_smallest.argtypes = [p, ctypes.c_int, i64, i64, p, p, p]
         L.w4a16_quantize.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_get_device_error.argtypes = [p]
         L.w4a16_selftest_wait_timeout.argtypes = [i64, p]
         L.w4a16_status_string.argtypes = [ctypes.c_int]
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
-        for f in ("w4a16_linear", "w4a16_linear_fused", "w4a16_linear_stack", "w4a16_dequant", "w4a16_quantize",
+        for f in ("w4a16_linear", "w4a16_linear_fused", "w4a16_linear_stack",
+                  "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_dequant", "w4a16_quantize",
                   "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
@@ -154,6 +157,32 @@ def make_layer_array(layers) -> ctypes.Array:
 
 def linear_stack_array(arr: ctypes.Array, M: int, g: int = 128, stream=None) -> None:
     _check("w4a16_linear_stack", lib().w4a16_linear_stack(arr, len(arr), M, g, _stream(stream)))
+
+
+def gather_rows(src: torch.Tensor, index: torch.Tensor, out=None, stream=None) -> torch.Tensor:
+    """dst[p] = src[index[p]] for bf16 rows; index int32 (include/w4a16.h)."""
+    rows, D = src.shape
+    P = index.shape[0]
+    if out is None:
+        out = torch.empty((P, D), dtype=torch.bfloat16, device=src.device)
+    _need_cuda(src, index, out)
+    assert src.dtype == torch.bfloat16 and index.dtype == torch.int32
+    _check("w4a16_gather_rows", lib().w4a16_gather_rows(src.data_ptr(), rows, D, index.data_ptr(),
+                                                        P, out.data_ptr(), _stream(stream)))
+    return out
+
+
+def topk_smallest(scores: torch.Tensor, k: int, stream=None):
+    """(int32 indices [k], fp32 scores [k]) of the k smallest scores (fp32 or
+    bf16), ascending by totalOrder, NaN last, ties by index."""
+    n = scores.shape[0]
+    _need_cuda(scores)
+    bits = {torch.float32: 32, torch.bfloat16: 16}[scores.dtype]
+    idx = torch.empty(k, dtype=torch.int32, device=scores.device)
+    val = torch.empty(k, dtype=torch.float32, device=scores.device)
+    _check("w4a16_topk_smallest", lib().w4a16_topk_smallest(
+        scores.data_ptr(), bits, n, k, idx.data_ptr(), val.data_ptr(), _stream(stream)))
+    return idx, val
 
 
 def dequant(w_packed: torch.Tensor, scales: torch.Tensor, g: int = 128, out=None,

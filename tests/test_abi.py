@@ -80,3 +80,18 @@ def test_dequant_and_quantize_reject_bad_args(L):
 def test_fused_rejects_before_launch(L, bias, res, out, N, act, want):
     assert L.w4a16_linear_fused(A, 2 * A, 3 * A, bias or None, res or None, out, 4, N, 256, 128,
                                 act, None) == want
+
+
+def test_readout_rejects_before_launch(L):
+    # gather: null, zero sizes, misaligned, dst overlapping src
+    assert L.w4a16_gather_rows(0, 4, 8, 2 * A, 2, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_gather_rows(A, 0, 8, 2 * A, 2, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_gather_rows(A, 4, 8, 2 * A + 4, 2, 3 * A, None) == W.ERR_ALIGNMENT
+    assert L.w4a16_gather_rows(A, 4, 8, 2 * A, 2, A + 16, None) == W.ERR_INVALID_ARG
+    # top-k: bad score width, k out of range, k above the supported limit, overlap
+    assert L.w4a16_topk_smallest(A, 8, 100, 10, 2 * A, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_topk_smallest(A, 32, 100, 0, 2 * A, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_topk_smallest(A, 32, 100, 101, 2 * A, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_topk_smallest(A, 32, 5000, 1025, 2 * A, 3 * A, None) == W.ERR_UNSUPPORTED
+    assert L.w4a16_topk_smallest(A, 16, 100, 10, A + 16, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_topk_smallest(A, 32, 100, 10, 2 * A, 2 * A + 16, None) == W.ERR_INVALID_ARG
