@@ -60,6 +60,7 @@ def lib():
         L.oracle_gather_rows.argtypes = [p, i64, i64, p, i64, p]
         L.oracle_gather_rows.restype = ctypes.c_int
         L.oracle_topk_smallest.argtypes = [p, i64, i64, p, p, p]
+        L.oracle_attention_rows.argtypes = [p, i64, i64, i64, p, i64, i64, p, i64, p, p]
         L.oracle_max_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -193,6 +194,22 @@ def topk_smallest(scores: np.ndarray, k: int):
     taken = np.empty(max(n, 1), dtype=np.uint8)
     lib().oracle_topk_smallest(_ptr(scores), n, k, _ptr(idx), _ptr(val), _ptr(taken))
     return idx, val
+
+
+def attention_rows(qkv_bits: np.ndarray, H: int, d: int, seq_start, window: int,
+                   rows=None) -> np.ndarray:
+    """fp64 attention outputs [len(rows), H d] for query tokens `rows` of the
+    packed batch: causal within each sequence [seq_start[s], seq_start[s+1])
+    and within a window of `window` tokens; qkv bf16 bits [M, 3 H d]."""
+    qkv_bits = np.ascontiguousarray(qkv_bits, dtype=np.uint16)
+    M = qkv_bits.shape[0]
+    st = np.ascontiguousarray(seq_start, dtype=np.int64)
+    rows = np.arange(M, dtype=np.int64) if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    out = np.empty((rows.shape[0], H * d), dtype=np.float64)
+    scratch = np.empty(max(1, min(M, window)), dtype=np.float64)
+    lib().oracle_attention_rows(_ptr(qkv_bits), M, H, d, _ptr(st), st.shape[0] - 1, window,
+                                _ptr(rows), rows.shape[0], _ptr(out), _ptr(scratch))
+    return out
 
 
 def max_threads() -> int:

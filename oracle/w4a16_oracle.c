@@ -283,6 +283,56 @@ void oracle_topk_smallest(const float* scores, int64_t n, int64_t k, int32_t* ou
     }
 }
 
+/* ---- attention prefill over packed sequences --------------------------------
+ *
+ * The decoder's attention between the QKV and output projections: causal
+ * within each protein-ligand pair's packed token sequence, limited to a
+ * sliding window of W tokens (the model's 32K window, Sec. 2.1).  Readings:
+ * standard multi-head scaled dot-product attention; qkv is the fused QKV
+ * projection output [M, 3 H d] (bf16) with q of head h in columns h d ..,
+ * k at H d + h d, v at 2 H d + h d; sequence s holds tokens
+ * [seq_start[s], seq_start[s+1]); query i attends to keys j of its own
+ * sequence with i - W < j <= i:
+ *   o[i, h, :] = sum_j softmax_j(q_i . k_j / sqrt(d)) v_j     (fp64)
+ * out: fp64 [M, H d] for the listed query tokens (rows). */
+void oracle_attention_rows(const uint16_t* qkv, int64_t M, int64_t H, int64_t d,
+                           const int64_t* seq_start, int64_t nseq, int64_t window,
+                           const int64_t* rows, int64_t nrows, double* out, double* scratch) {
+    (void)M;
+    const int64_t ld = 3 * H * d;
+    const double scale = 1.0 / sqrt((double)d);
+    for (int64_t r = 0; r < nrows; ++r) {
+        const int64_t i = rows[r];
+        int64_t s = 0;
+        while (s + 1 < nseq && seq_start[s + 1] <= i) ++s;
+        const int64_t lo0 = seq_start[s];
+        const int64_t lo = i - window + 1 > lo0 ? i - window + 1 : lo0;
+        for (int64_t h = 0; h < H; ++h) {
+            const uint16_t* q = qkv + i * ld + h * d;
+            double mx = -INFINITY;
+            for (int64_t j = lo; j <= i; ++j) {
+                const uint16_t* k = qkv + j * ld + H * d + h * d;
+                double dot = 0.0;
+                for (int64_t t = 0; t < d; ++t)
+                    dot += (double)oracle_bf16_to_f32(q[t]) * (double)oracle_bf16_to_f32(k[t]);
+                scratch[j - lo] = dot * scale;
+                if (scratch[j - lo] > mx) mx = scratch[j - lo];
+            }
+            double den = 0.0;
+            for (int64_t j = lo; j <= i; ++j) {
+                scratch[j - lo] = exp(scratch[j - lo] - mx);
+                den += scratch[j - lo];
+            }
+            for (int64_t t = 0; t < d; ++t) {
+                double acc = 0.0;
+                for (int64_t j = lo; j <= i; ++j)
+                    acc += scratch[j - lo] * (double)oracle_bf16_to_f32(qkv[j * ld + 2 * H * d + h * d + t]);
+                out[r * H * d + h * d + t] = acc / den;
+            }
+        }
+    }
+}
+
 int oracle_max_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

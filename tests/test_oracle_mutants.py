@@ -6,7 +6,9 @@ truncating bf16 rounding, fp32 accumulation, wrong activation row, and in
 the fused epilogue swapped gate/up, a wrong SiLU sign, the tanh GELU
 approximation, a wrong residual row, bias after the activation; in the
 readout top-k ties by the last index, unordered zeros, NaN first, and a gather
-that does not zero the rows of bad indices), points
+that does not zero the rows of bad indices; in attention a dropped 1/sqrt(d),
+a window one token too wide, values read from the keys, and keys of other
+sequences), points
 the oracle module at it and runs the pins: at least one must fail.  The
 mistakes live only in temporary copies on the CPU."""
 import ctypes
@@ -40,6 +42,11 @@ MUTANTS = {
                                  "return ia > ib ? -1 : (ia < ib ? 1 : 0);")],
     "topk_zeros_unordered": [("if (sa != sb) return sa ? -1 : 1;", "(void)sa; (void)sb;")],
     "topk_nan_first": [("if (na != nb) return na ? 1 : -1;", "if (na != nb) return na ? -1 : 1;")],
+    "attention_no_scale": [("scratch[j - lo] = dot * scale;", "scratch[j - lo] = dot;")],
+    "attention_window_off_by_one": [("i - window + 1 > lo0 ? i - window + 1 : lo0",
+                                     "i - window > lo0 ? i - window : lo0")],
+    "attention_v_from_k": [("qkv[j * ld + 2 * H * d + h * d + t]", "qkv[j * ld + H * d + h * d + t]")],
+    "attention_ignores_sequences": [("const int64_t lo0 = seq_start[s];", "const int64_t lo0 = 0;")],
     "gather_bad_rows_not_zeroed": [("for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 0;",
                                     "for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 1;")],
 }
@@ -65,6 +72,10 @@ PINS = [
     P.test_gather_rows_by_hand,
     P.test_topk_hand_example_ties_zeros_nan,
     P.test_topk_matches_a_textbook_sort,
+    P.test_attention_single_key_and_window_one_return_v,
+    P.test_attention_equal_scores_give_the_mean,
+    P.test_attention_two_keys_closed_form,
+    P.test_attention_is_causal_and_sequences_are_independent,
 ]
 
 
@@ -90,7 +101,7 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
         for fn in ("oracle_bf16_rne", "oracle_bf16_to_f32", "oracle_unpack", "oracle_pack",
                    "oracle_quantize", "oracle_dequant", "oracle_linear_rows",
                    "oracle_linear_points", "oracle_epilogue_rows", "oracle_gather_rows",
-                   "oracle_topk_smallest", "oracle_max_threads"):
+                   "oracle_topk_smallest", "oracle_attention_rows", "oracle_max_threads"):
             getattr(mut, fn).argtypes = getattr(good, fn).argtypes
             getattr(mut, fn).restype = getattr(good, fn).restype
         monkeypatch.setattr(O, "_lib", mut)

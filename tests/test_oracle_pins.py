@@ -386,3 +386,63 @@ def test_topk_matches_a_textbook_sort():
         idx, val = O.topk_smallest(s, k)
         assert idx.tolist() == order[:k]
         assert val.tobytes() == s[order[:k]].tobytes()
+
+
+# ---- attention prefill over packed sequences (causal per sequence, sliding
+# window; Sec. 2.1's 32K window) ---------------------------------------------
+
+def _qkv(M, H, d, seed, q_zero=False):
+    rng = np.random.default_rng(seed)
+    a = rng.normal(size=(M, 3 * H * d)).astype(np.float32)
+    if q_zero:
+        a[:, :H * d] = 0.0
+    return O.bf16_rne_array(a)
+
+
+def test_attention_single_key_and_window_one_return_v():
+    H, d = 2, 8
+    qkv = _qkv(10, H, d, 1)
+    v = O.bf16_bits_to_f32(qkv[:, 2 * H * d:]).astype(np.float64)
+    out = O.attention_rows(qkv, H, d, [0, 4, 10], window=1 << 15)
+    assert np.array_equal(out[0], v[0]) and np.array_equal(out[4], v[4])   # first of each sequence
+    out1 = O.attention_rows(qkv, H, d, [0, 4, 10], window=1)               # only itself
+    assert np.array_equal(out1, v)
+
+
+def test_attention_equal_scores_give_the_mean():
+    H, d = 1, 16
+    qkv = _qkv(9, H, d, 2, q_zero=True)          # q = 0: every score is 0
+    v = O.bf16_bits_to_f32(qkv[:, 2 * d:]).astype(np.float64)
+    out = O.attention_rows(qkv, H, d, [0, 9], window=4)
+    for i in range(9):
+        lo = max(0, i - 3)
+        assert np.allclose(out[i], v[lo:i + 1].mean(axis=0), rtol=0, atol=1e-14)
+
+
+def test_attention_two_keys_closed_form():
+    # d = 4 (scale 1/2): q1 = e0, k0 = 0, k1 = 2 e0 -> scores 0 and 1, weights 1:e
+    H, d = 1, 4
+    qkv = np.zeros((2, 12), dtype=np.uint16)
+    qkv[1, 0] = 0x3F80                           # q1[0] = 1
+    qkv[1, 4] = 0x4000                           # k1[0] = 2
+    qkv[0, 8:12] = [0x3F80, 0x4000, 0xBF80, 0]   # v0 = (1, 2, -1, 0)
+    qkv[1, 8:12] = [0x4040, 0, 0x3F00, 0x4080]   # v1 = (3, 0, 0.5, 4)
+    out = O.attention_rows(qkv, H, d, [0, 2], window=8)
+    e = math.e
+    want = (np.array([1, 2, -1, 0]) + e * np.array([3, 0, 0.5, 4])) / (1 + e)
+    assert np.allclose(out[1], want, rtol=0, atol=1e-15)
+
+
+def test_attention_is_causal_and_sequences_are_independent():
+    H, d = 2, 8
+    qkv = _qkv(12, H, d, 3)
+    st = [0, 5, 12]
+    base = O.attention_rows(qkv, H, d, st, window=64)
+    later = qkv.copy()
+    later[8:, H * d:] = O.bf16_rne_array(np.full((4, 2 * H * d), 7.0, dtype=np.float32))
+    moved = O.attention_rows(later, H, d, st, window=64)
+    assert np.array_equal(moved[:8], base[:8])     # keys/values after a query do not matter
+    other = qkv.copy()
+    other[:5] = O.bf16_rne_array(np.full((5, 3 * H * d), -3.0, dtype=np.float32))
+    iso = O.attention_rows(other, H, d, st, window=64)
+    assert np.array_equal(iso[5:], base[5:])       # another sequence does not matter
