@@ -153,6 +153,32 @@ int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales_bf16,
                    int64_t N, int64_t K, int64_t g, void* stream);
 
 /*
+ * Attention prefill over a packed batch of sequences: the decoder's
+ * attention between the QKV and output projections, causal within each
+ * protein-ligand pair's token sequence and limited to a sliding window of
+ * `window` tokens (the model's 32K window, Sec. 2.1); the paper gives no
+ * further detail, so this is standard multi-head scaled dot-product
+ * attention:
+ *   out[i, h*d + t] = sum_j softmax_j(q_i . k_j / sqrt(d)) v_j[t]
+ * over keys j of i's sequence with i - window < j <= i.
+ *   qkv_bf16       [M, 3*H*d] bf16, device: the fused QKV projection output;
+ *                  q of head h in columns h*d .., k at H*d + h*d, v at
+ *                  2*H*d + h*d
+ *   seq_start_i32  [nseq + 1] int32, device: sequence s is tokens
+ *                  [seq_start[s], seq_start[s+1]); nondecreasing, within
+ *                  [0, M] (else nothing is written and W4A16_ERR_INVALID_ARG
+ *                  is recorded in the device status word); tokens outside
+ *                  every sequence are left untouched in out
+ *   d              head dimension, 128 (else W4A16_ERR_UNSUPPORTED)
+ *   out_bf16       [M, H*d] bf16, device, must not overlap the inputs
+ * The softmax is computed in fp32 with P rounded to bf16 for the PV product
+ * (tcgen05), O accumulated in fp32, one bf16 rounding at the store.
+ */
+int w4a16_attention_prefill(const void* qkv_bf16, const void* seq_start_i32, int64_t nseq,
+                            int64_t M, int64_t H, int64_t d, int64_t window, void* out_bf16,
+                            void* stream);
+
+/*
  * Scoring readout, the last modules of the screening pipeline (Sec. 3.3):
  * the affinity head reads one hidden state per pair of the packed batch
  * (w4a16_gather_rows, then w4a16_linear_fused with the head's weights and

@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <cmath>
 #include <cstdlib>
 #include <mutex>
 
@@ -329,6 +330,42 @@ extern "C" int w4a16_quantize(const void* w_f32, void* w_packed_u8, void* scales
     return launch_quantize(static_cast<const float*>(w_f32), static_cast<uint8_t*>(w_packed_u8),
                            static_cast<uint16_t*>(scales_bf16), N, K, g,
                            static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_attention_prefill(const void* qkv_bf16, const void* seq_start_i32,
+                                       int64_t nseq, int64_t M, int64_t H, int64_t d,
+                                       int64_t window, void* out_bf16, void* stream) {
+    if (qkv_bf16 == nullptr || seq_start_i32 == nullptr || out_bf16 == nullptr)
+        return W4A16_ERR_INVALID_ARG;
+    if (nseq <= 0 || M <= 0 || H <= 0 || d <= 0 || window <= 0) return W4A16_ERR_INVALID_ARG;
+    if (d != attention_head_dim()) return W4A16_ERR_UNSUPPORTED;
+    if (M > kMaxDim || nseq > kMaxDim / 2 || H > 65535 || 3 * H * d > kMaxDim)
+        return W4A16_ERR_UNSUPPORTED;
+    if (!aligned16(qkv_bf16) || !aligned16(seq_start_i32) || !aligned16(out_bf16))
+        return W4A16_ERR_ALIGNMENT;
+    const int64_t out_bytes = M * H * d * 2;
+    if (overlaps(out_bf16, out_bytes, qkv_bf16, M * 3 * H * d * 2) ||
+        overlaps(out_bf16, out_bytes, seq_start_i32, (nseq + 1) * 4))
+        return W4A16_ERR_INVALID_ARG;
+    DeviceState* st = nullptr;
+    int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    alignas(64) CUtensorMap tq;
+    rc = encode_2d(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, qkv_bf16, 3 * H * d, M, 3 * H * d * 2,
+                   64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != W4A16_OK) return rc;
+    AttnParams p;
+    p.seq_start = static_cast<const int32_t*>(seq_start_i32);
+    p.out = static_cast<uint16_t*>(out_bf16);
+    p.status = st->status;
+    p.M = static_cast<int>(M);
+    p.H = static_cast<int>(H);
+    p.nseq = static_cast<int>(nseq);
+    p.window = window > kMaxDim ? static_cast<int>(kMaxDim) : static_cast<int>(window);
+    p.scale = 1.0f / sqrtf(static_cast<float>(d));
+    return launch_attention_prefill(&tq, p, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? W4A16_OK
                : W4A16_ERR_CUDA;
 }

@@ -1,0 +1,424 @@
+// Attention prefill over packed sequences for sm_103a: the decoder's
+// attention between the QKV and output projections, causal within each
+// protein-ligand pair's sequence and limited to a sliding window (the
+// model's 32K window, Sec. 2.1).
+//
+//   o[i, h, :] = sum_j softmax_j(q_i . k_j / sqrt(d)) v_j,
+//   j in the sequence of i, i - W < j <= i;  d = 128.
+//
+// One CTA per (128-query block, head), flash-attention style on the
+// 5th-generation tensor core:
+//   S  = Q K^T   tcgen05.mma kind::f16, A = Q and B = K from shared memory
+//                (TMA, 128-byte swizzle, K-major), S fp32 in tensor memory;
+//   softmax      four warps, thread = query row: tcgen05.ld of its S row,
+//                mask, running max and sum in fp32 (exp2 with the scale
+//                folded in), P as bf16 pairs written back into tensor memory
+//                with tcgen05.st; O rescaled in tensor memory when the
+//                running max grows;
+//   O += P V     tcgen05.mma with A = P from tensor memory and B = V from
+//                shared memory as an MN-major operand (V is stored token-
+//                major, d contiguous -- exactly the layout the TMA box has);
+//   epilogue     O / l, bf16, 16-byte stores.
+// The MMA warp issues S of the next key block as soon as the softmax warps
+// have read S, so the softmax of block j+1 overlaps the PV product of block
+// j.  K/V blocks stream through a two-stage TMA ring.
+// Every wait is bounded (ptx.cuh); on a timeout the kernel records
+// W4A16_ERR_TIMEOUT, waits for its own copies and MMAs and frees tensor memory.
+#include "internal.h"
+#include "ptx.cuh"
+
+#include <cuda_bf16.h>
+
+namespace w4a16 {
+
+namespace {
+
+constexpr int kD = 128;        // head dimension
+constexpr int kBQ = 128;       // queries per CTA (MMA M)
+constexpr int kBKV = 128;      // keys per block (MMA N of S, K of PV)
+constexpr int kKVStages = 2;
+constexpr int kThreads = 6 * 32;  // TMA warp, MMA warp, 4 softmax warps
+
+struct AttnLayout {
+    static constexpr int BOX = kBQ * 64 * 2;       // one [128 rows x 64 cols] bf16 box: 16 KB
+    static constexpr int TILE = 2 * BOX;           // [128 x 128]: 32 KB
+    static constexpr int Q_OFF = 0;
+    static constexpr int K_OFF = Q_OFF + TILE;
+    static constexpr int V_OFF = K_OFF + kKVStages * TILE;
+    static constexpr int BAR_OFF = V_OFF + kKVStages * TILE;
+    // q_full, kv_full[S], kv_empty[S], s_full, s_free, p_full, o_ready, drain
+    static constexpr int NBARS = 1 + 2 * kKVStages + 5;
+    static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
+    static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
+    // tensor memory columns
+    static constexpr int S_COL = 0, P_COL = 128, O_COL = 256, TMEM_COLS = 512;
+};
+
+// SS MMA: D[tmem] (+)= A[smem] * B[smem]^T, kind::f16.
+__device__ __forceinline__ void tc_mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Shared-memory descriptor of an MN-major operand with the 128-byte swizzle:
+// 128-byte rows of 64 MN-contiguous elements, one row per K index, 8-row
+// (1024-byte) swizzle atoms; the next 8 K rows are `sbo` bytes on, the next
+// 64 MN elements `lbo` bytes on.
+__device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr, uint32_t lbo,
+                                                        uint32_t sbo) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+    d |= static_cast<uint64_t>((lbo & 0x3FFFFu) >> 4) << 16;
+    d |= static_cast<uint64_t>((sbo & 0x3FFFFu) >> 4) << 32;
+    d |= static_cast<uint64_t>(1) << 46;
+    d |= static_cast<uint64_t>(2) << 61;
+    return d;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+constexpr float kMaskedScore = -1.0e30f;  // finite: fully masked rows stay NaN-free
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p) {
+    using L = AttnLayout;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t sbase = (raw + 1023u) & ~1023u;
+    uint8_t* smem = smem_raw + (sbase - raw);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // ---- which (sequence, query block) this CTA takes: blocks of sequence s
+    // are numbered from its last (the heaviest under the causal mask) down
+    __shared__ int job[4];  // seq start, seq end, first query, valid
+    if (warp == 0) {
+        const int x = blockIdx.x;
+        int base = 0, found = 0, ss = 0, se = 0, q0 = 0, bad = 0;
+        for (int s0 = 0; s0 < p.nseq && !found; s0 += 32) {
+            const int s = s0 + lane;
+            int a = 0, b = 0, nqb = 0;
+            if (s < p.nseq) {
+                a = p.seq_start[s];
+                b = p.seq_start[s + 1];
+                if (a < 0 || b < a || b > p.M) bad = 1;
+                nqb = b > a ? (b - a + kBQ - 1) / kBQ : 0;
+            }
+            if (__any_sync(0xffffffffu, bad)) {
+                bad = 1;
+                break;
+            }
+            int incl = nqb;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += t;
+            }
+            const int excl = incl - nqb;
+            const bool mine = s < p.nseq && x >= base + excl && x < base + incl;
+            const unsigned who = __ballot_sync(0xffffffffu, mine);
+            if (who) {
+                const int src = __ffs(who) - 1;
+                const int e = __shfl_sync(0xffffffffu, excl, src);
+                const int n = __shfl_sync(0xffffffffu, nqb, src);
+                ss = __shfl_sync(0xffffffffu, a, src);
+                se = __shfl_sync(0xffffffffu, b, src);
+                const int local = x - base - e;
+                q0 = ss + (n - 1 - local) * kBQ;
+                found = 1;
+            }
+            base += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) {
+            if (bad) atomicExch(p.status, 1 /* W4A16_ERR_INVALID_ARG */);
+            job[0] = ss;
+            job[1] = se;
+            job[2] = q0;
+            job[3] = found && !bad;
+        }
+    }
+    __syncthreads();
+    if (!job[3]) return;  // past the last query block (the grid is an upper bound)
+    const int ss = job[0], se = job[1], q0 = job[2];
+    const int h = blockIdx.y;
+    const int W = p.window;
+    // key blocks of the sequence that any query of the block can see
+    const int q_last = (q0 + kBQ - 1 < se - 1 ? q0 + kBQ - 1 : se - 1);
+    const int k_first = q0 - W + 1 > ss ? q0 - W + 1 : ss;
+    const int b_first = (k_first - ss) / kBKV, b_last = (q_last - ss) / kBKV;
+    const int nblk = b_last - b_first + 1;
+
+    const uint32_t bars = sbase + L::BAR_OFF;
+    const uint32_t q_full = bars;
+    auto kv_full = [&](int s) { return bars + 8u * (1 + s); };
+    auto kv_empty = [&](int s) { return bars + 8u * (1 + kKVStages + s); };
+    const uint32_t s_full = bars + 8u * (1 + 2 * kKVStages);
+    const uint32_t s_free = s_full + 8u;
+    const uint32_t p_full = s_full + 16u;
+    const uint32_t o_ready = s_full + 24u;
+    const uint32_t drain = s_full + 32u;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
+
+    if (threadIdx.x == 0) {
+        mbar_init(q_full, 1);
+        for (int s = 0; s < kKVStages; ++s) {
+            mbar_init(kv_full(s), 1);
+            mbar_init(kv_empty(s), 1);
+        }
+        mbar_init(s_full, 1);
+        mbar_init(s_free, 4);   // one arrival per softmax warp
+        mbar_init(p_full, 4);
+        mbar_init(o_ready, 1);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap_qkv);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int Hd = p.H * kD;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            bool ok = true;
+            mbar_arrive_expect_tx(q_full, L::TILE);
+            tma_load_2d(sbase + L::Q_OFF, &tmap_qkv, q_full, h * kD, q0);
+            tma_load_2d(sbase + L::Q_OFF + L::BOX, &tmap_qkv, q_full, h * kD + 64, q0);
+            int j = 0;
+            for (; ok && j < nblk; ++j) {
+                const int s = j % kKVStages;
+                if (!wait_one(kv_empty(s), ((j / kKVStages) & 1u) ^ 1u, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
+                const int row = ss + (b_first + j) * kBKV;
+                mbar_arrive_expect_tx(kv_full(s), 2 * L::TILE);
+                const uint32_t ks = sbase + L::K_OFF + s * L::TILE;
+                const uint32_t vs = sbase + L::V_OFF + s * L::TILE;
+                tma_load_2d(ks, &tmap_qkv, kv_full(s), Hd + h * kD, row);
+                tma_load_2d(ks + L::BOX, &tmap_qkv, kv_full(s), Hd + h * kD + 64, row);
+                tma_load_2d(vs, &tmap_qkv, kv_full(s), 2 * Hd + h * kD, row);
+                tma_load_2d(vs + L::BOX, &tmap_qkv, kv_full(s), 2 * Hd + h * kD + 64, row);
+            }
+            // every load issued has landed before exit
+            {
+                const uint64_t t0 = global_timer_ns();
+                while (!mbar_try_wait(q_full, 0)) {
+                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
+                }
+            }
+            const int last = j < kKVStages ? j : kKVStages;
+            for (int i = j - last; i < j; ++i) {
+                const uint64_t t0 = global_timer_ns();
+                while (!mbar_try_wait(kv_full(i % kKVStages), (i / kKVStages) & 1u)) {
+                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
+            constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
+            bool ok = wait_one(q_full, 0, abort_flag, p.status);
+            auto issue_s = [&](int j) -> bool {
+                const int s = j % kKVStages;
+                if (!wait_one(kv_full(s), (j / kKVStages) & 1u, abort_flag, p.status)) return false;
+                // S may be overwritten once the softmax warps have read block j-1
+                if (j > 0 && !wait_one(s_free, (j - 1) & 1u, abort_flag, p.status)) return false;
+                tc_fence_after();
+                const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + s * L::TILE;
+#pragma unroll
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
+                    tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
+                              sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(s_full);
+                return true;
+            };
+            if (ok && nblk > 0) ok = issue_s(0);
+            for (int j = 0; ok && j < nblk; ++j) {
+                if (j + 1 < nblk && !issue_s(j + 1)) {
+                    ok = false;
+                    break;
+                }
+                // O += P V once the softmax warps have written P of block j
+                if (!wait_one(p_full, j & 1u, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int s = j % kKVStages;
+                const uint32_t vs = sbase + L::V_OFF + s * L::TILE;
+#pragma unroll
+                for (int kk = 0; kk < kBKV / 16; ++kk) {
+                    // keys 16 kk .. 16 kk + 15: rows of the V tile; P columns 8 kk ..
+                    tc_mma_ts(tmem + L::O_COL, tmem + L::P_COL + kk * 8,
+                              sdesc_mnmajor_sw128(vs + kk * 16 * 128, L::BOX, 1024), idesc_o,
+                              (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc_commit(o_ready);
+                tc_commit(kv_empty(s));
+            }
+            tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
+            const uint64_t t0 = global_timer_ns();
+            while (!mbar_try_wait(drain, 0)) {
+                if (global_timer_ns() - t0 > kWaitLimitNs) break;
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ softmax + epilogue
+        const int sub = warp & 3;  // TMEM sub-partition: lanes 32 sub ..
+        const int r = sub * 32 + lane;          // query row within the block
+        const int i = q0 + r;                   // query token
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
+        const float c = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
+        float m = kMaskedScore, l = 0.0f;
+        bool ok = true;
+        for (int j = 0; ok && j < nblk; ++j) {
+            if (!wait_warp(s_full, j & 1u, abort_flag, p.status)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const int kbase = ss + (b_first + j) * kBKV;
+            float sv[kBKV];
+#pragma unroll
+            for (int ch = 0; ch < kBKV / 32; ++ch) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(lane_base + L::S_COL + ch * 32, v);
+                tmem_ld_wait(v);
+#pragma unroll
+                for (int t = 0; t < 32; ++t) {
+                    const int key = kbase + ch * 32 + t;
+                    const bool allowed = key <= i && key > i - W && key < se;
+                    sv[ch * 32 + t] = allowed ? __uint_as_float(v[t]) * c : kMaskedScore;
+                }
+            }
+            // S is in registers: the next block's S MMA may start
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(s_free);
+            float mb = kMaskedScore;
+#pragma unroll
+            for (int t = 0; t < kBKV; ++t) mb = fmaxf(mb, sv[t]);
+            const float m_new = fmaxf(m, mb);
+            const float alpha = ex2(m - m_new);
+            float sum = 0.0f;
+            uint32_t pk[kBKV / 2];
+#pragma unroll
+            for (int t = 0; t < kBKV / 2; ++t) {
+                // masked keys get exactly 0 (a row may have none allowed in a block)
+                const float p0 = sv[2 * t] > kMaskedScore ? ex2(sv[2 * t] - m_new) : 0.0f;
+                const float p1 = sv[2 * t + 1] > kMaskedScore ? ex2(sv[2 * t + 1] - m_new) : 0.0f;
+                sum += p0 + p1;
+                pk[t] = pack_bf16x2_rn(p0, p1);
+            }
+            l = l * alpha + sum;
+            m = m_new;
+            // P and O of block j-1 are in use until its PV product completes
+            if (j > 0) {
+                if (!wait_warp(o_ready, (j - 1) & 1u, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, alpha < 1.0f)) {
+#pragma unroll 1
+                    for (int ch = 0; ch < kD / 32; ++ch) {
+                        uint32_t v[32];
+                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
+                        tmem_ld_wait(v);
+#pragma unroll
+                        for (int t = 0; t < 32; ++t)
+                            v[t] = __float_as_uint(__uint_as_float(v[t]) * alpha);
+                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
+                    }
+                }
+            }
+            uint32_t half[32];
+#pragma unroll
+            for (int t = 0; t < 32; ++t) half[t] = pk[t];
+            tmem_st_32x32b_x32(lane_base + L::P_COL, half);
+#pragma unroll
+            for (int t = 0; t < 32; ++t) half[t] = pk[32 + t];
+            tmem_st_32x32b_x32(lane_base + L::P_COL + 32, half);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(p_full);
+        }
+        // ---- epilogue: O / l -> bf16
+        if (ok && nblk > 0 && wait_warp(o_ready, (nblk - 1) & 1u, abort_flag, p.status)) {
+            tc_fence_after();
+            const float inv = l > 0.0f ? 1.0f / l : 0.0f;
+            __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out) +
+                                  static_cast<int64_t>(i) * Hd + h * kD;
+#pragma unroll 1
+            for (int ch = 0; ch < kD / 32; ++ch) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
+                tmem_ld_wait(v);
+                if (i < se) {
+                    uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 w;
+                        w.x = pack_bf16x2_rn(__uint_as_float(v[8 * q + 0]) * inv, __uint_as_float(v[8 * q + 1]) * inv);
+                        w.y = pack_bf16x2_rn(__uint_as_float(v[8 * q + 2]) * inv, __uint_as_float(v[8 * q + 3]) * inv);
+                        w.z = pack_bf16x2_rn(__uint_as_float(v[8 * q + 4]) * inv, __uint_as_float(v[8 * q + 5]) * inv);
+                        w.w = pack_bf16x2_rn(__uint_as_float(v[8 * q + 6]) * inv, __uint_as_float(v[8 * q + 7]) * inv);
+                        dst[q] = w;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
+}
+
+}  // namespace
+
+cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnParams& p,
+                                     cudaStream_t stream) {
+    using L = AttnLayout;
+    cudaError_t e = cudaFuncSetAttribute(attention_prefill_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         L::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    // upper bound on the query blocks: sum over sequences of ceil(len / 128)
+    const int64_t qblocks = (static_cast<int64_t>(p.M) + kBQ - 1) / kBQ + p.nseq;
+    const dim3 grid(static_cast<unsigned>(qblocks), static_cast<unsigned>(p.H));
+    attention_prefill_kernel<<<grid, kThreads, L::SMEM_BYTES, stream>>>(*tmap_qkv, p);
+    return cudaGetLastError();
+}
+
+int attention_head_dim() { return kD; }
+
+}  // namespace w4a16

@@ -63,6 +63,18 @@ int gemv_tokens_per_tile(int64_t M);
 cudaError_t gemv_launch(const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                         const GemvParams& p, int sm_count, cudaStream_t stream);
 
+// Attention prefill over packed sequences (attention.cu).
+struct AttnParams {
+    const int32_t* seq_start;  // device [nseq + 1]
+    uint16_t* out;             // bf16 bits [M, H * 128]
+    int* status;
+    int M, H, nseq, window;
+    float scale;               // 1 / sqrt(head dim)
+};
+int attention_head_dim();
+cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnParams& p,
+                                     cudaStream_t stream);
+
 // Scoring readout (readout.cu).
 constexpr int kTopkMaxK = 1024;  // largest k of the top-k
 cudaError_t launch_topk_smallest(const void* scores, bool bf16, int64_t n, int k,

@@ -54,6 +54,7 @@ def lib() -> ctypes.CDLL:
         L.w4a16_linear_stack.argtypes = [ctypes.POINTER(Layer), i64, i64, i64, p]
         L.w4a16_dequant.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_gather_rows.argtypes = [p, i64, i64, p, i64, p, p]
+        L.w4a16_attention_prefill.argtypes = [p, p, i64, i64, i64, i64, i64, p, p]
         L.w4a16_topk_smallest.argtypes = [p, ctypes.c_int, i64, i64, p, p, p]
         L.w4a16_quantize.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_get_device_error.argtypes = [p]
@@ -62,7 +63,7 @@ def lib() -> ctypes.CDLL:
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
         for f in ("w4a16_linear", "w4a16_linear_fused", "w4a16_linear_stack",
-                  "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_dequant", "w4a16_quantize",
+                  "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_attention_prefill", "w4a16_dequant", "w4a16_quantize",
                   "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
@@ -157,6 +158,22 @@ def make_layer_array(layers) -> ctypes.Array:
 
 def linear_stack_array(arr: ctypes.Array, M: int, g: int = 128, stream=None) -> None:
     _check("w4a16_linear_stack", lib().w4a16_linear_stack(arr, len(arr), M, g, _stream(stream)))
+
+
+def attention_prefill(qkv: torch.Tensor, seq_start: torch.Tensor, H: int, window: int = 32768,
+                      out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Causal sliding-window attention over packed sequences (include/w4a16.h):
+    qkv bf16 [M, 3 H 128], seq_start int32 [nseq + 1] -> out bf16 [M, H 128]."""
+    M = qkv.shape[0]
+    d = qkv.shape[1] // (3 * H)
+    if out is None:
+        out = torch.zeros((M, H * d), dtype=torch.bfloat16, device=qkv.device)
+    _need_cuda(qkv, seq_start, out)
+    assert qkv.dtype == torch.bfloat16 and seq_start.dtype == torch.int32
+    _check("w4a16_attention_prefill", lib().w4a16_attention_prefill(
+        qkv.data_ptr(), seq_start.data_ptr(), seq_start.shape[0] - 1, M, H, d, int(window),
+        out.data_ptr(), _stream(stream)))
+    return out
 
 
 def gather_rows(src: torch.Tensor, index: torch.Tensor, out=None, stream=None) -> torch.Tensor:

@@ -95,3 +95,11 @@ def test_readout_rejects_before_launch(L):
     assert L.w4a16_topk_smallest(A, 32, 5000, 1025, 2 * A, 3 * A, None) == W.ERR_UNSUPPORTED
     assert L.w4a16_topk_smallest(A, 16, 100, 10, A + 16, 3 * A, None) == W.ERR_INVALID_ARG
     assert L.w4a16_topk_smallest(A, 32, 100, 10, 2 * A, 2 * A + 16, None) == W.ERR_INVALID_ARG
+
+
+def test_attention_rejects_before_launch(L):
+    assert L.w4a16_attention_prefill(0, 2 * A, 1, 64, 2, 128, 100, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_attention_prefill(A, 2 * A, 1, 64, 2, 64, 100, 3 * A, None) == W.ERR_UNSUPPORTED
+    assert L.w4a16_attention_prefill(A, 2 * A, 1, 64, 2, 128, 0, 3 * A, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_attention_prefill(A, 2 * A + 4, 1, 64, 2, 128, 9, 3 * A, None) == W.ERR_ALIGNMENT
+    assert L.w4a16_attention_prefill(A, 2 * A, 1, 64, 2, 128, 9, A + 64, None) == W.ERR_INVALID_ARG
