@@ -60,7 +60,7 @@ def kernel_source_hash(kind: str = "ts") -> str:
 
 
 def ncu_traffic(config: str, m: int):
-    if config == "topk":
+    if config in ("topk", "attention"):
         return None  # no capture of the readout kernels is summarised
     if config == "gemv":
         if m > 8:  # the capture is of the M <= 8 instantiation
@@ -280,6 +280,30 @@ class LinearWorkload:
             W.linear(self.x, packed, scales, self.g, out=self.out, stream=stream)
 
 
+class AttentionWorkload:
+    """Attention prefill of one layer over the packed batch: `pairs` sequences
+    of `tokens` tokens, 96 heads of 128, causal, 32K window; qkv resident."""
+
+    def __init__(self, pairs, tokens, heads, window, seed):
+        import torch
+        from paper_2608_30877_gb300 import synthetic as S
+        self.name = f"attention_{pairs}x{tokens}_h{heads}"
+        M = pairs * tokens
+        self.H, self.window = heads, window
+        self.x = S.make_x(M, 3 * heads * 128, seed, "cuda")
+        self.seq_start = torch.arange(0, M + 1, tokens, dtype=torch.int32, device="cuda")
+        self.out = torch.empty((M, heads * 128), dtype=torch.bfloat16, device="cuda")
+        keys = pairs * sum(min(i + 1, window) for i in range(tokens))  # allowed (i, j) pairs
+        self.flops = 4.0 * 128 * heads * keys          # QK^T and PV, 2 flops per MAC
+        self.bytes = 2.0 * M * 3 * heads * 128 + 2.0 * M * heads * 128
+        self.launches_per_step = 1
+
+    def step(self, stream=None):
+        from paper_2608_30877_gb300 import w4a16 as W
+        W.attention_prefill(self.x, self.seq_start, self.H, self.window, out=self.out,
+                            stream=stream)
+
+
 class TopkWorkload:
     """Result sorting of the screening set: the k best (smallest) of n
     predicted affinities, fp32 scores resident on the device."""
@@ -327,6 +351,29 @@ def oracle_sample(K: int, N_rows: int, target_s: float, rows_max: int = 2048):
         r = min(rows_max, max(r + 1, int(r * (target_s / 2) / max(dt, 1e-3))))
 
 
+def oracle_attention_sample(target_s: float = 10.0):
+    """Times the oracle's fp64 attention on query rows of one 1024-token
+    sequence with 96 heads of 128 (rows taken from the end, the longest),
+    growing the row count toward target_s; returns (TFLOP/s, description)."""
+    import numpy as np
+    from oracle import oracle as O
+    from paper_2608_30877_gb300 import synthetic as S
+    H, L = 96, 1024
+    bits = S.bf16_bits(S.make_x(L, 3 * H * 128, 9, "cpu"))
+    st = np.array([0, L], dtype=np.int64)
+    r = 1
+    while True:
+        rows = np.arange(L - r, L, dtype=np.int64)
+        t0 = time.perf_counter()
+        O.attention_rows(bits, H, 128, st, 32768, rows=rows)
+        dt = time.perf_counter() - t0
+        if dt >= target_s / 3 or r >= 256:
+            flops = 4.0 * 128 * H * float(np.sum(rows + 1))
+            return flops / dt / 1e12, (f"oracle fp64 attention, {r} query rows of a 1024-token "
+                                       f"sequence x 96 heads in {dt:.2f} s on 1 thread")
+        r = min(256, max(r + 1, int(r * (target_s / 2) / max(dt, 1e-3))))
+
+
 def oracle_topk_sample(n: int, k: int):
     """Times the oracle's top-k (plain repeated selection, one thread) on the
     same n seeded scores with k reduced to fit ~10 s; returns (GB/s of the
@@ -361,6 +408,11 @@ def config_for(args):
                 "pairs": args.pairs, "tokens_per_pair": 1024, "layers": args.layers, "g": 128,
                 "l2": "inputs larger than L2 (88 GB packed weights, >=1.6 GB activations per "
                       "linear); no flush"}
+    if c == "attention":
+        return {"workload": f"attention prefill, {args.pairs} pairs x 1024 tokens, 96 heads x 128, "
+                            "causal, window 32768",
+                "pairs": args.pairs, "tokens_per_pair": 1024, "heads": 96, "head_dim": 128,
+                "window": 32768, "l2": "qkv (4.8 GB at 64 pairs) larger than L2; no flush"}
     if c == "topk":
         return {"workload": f"top-k of predicted affinities, n={args.topk_n}, k={args.topk_k}",
                 "n": args.topk_n, "k": args.topk_k,
@@ -384,6 +436,26 @@ def run_reference(args):
     if rank != 0:
         return 0
     from paper_2608_30877_gb300 import synthetic as S
+    if args.config == "attention":
+        vals, desc = [], ""
+        for i in range(args.warmup + args.steps):
+            tf, desc = oracle_attention_sample(args.ref_seconds)
+            if i >= args.warmup:
+                vals.append(tf)
+        value = statistics.median(vals)
+        step_flops = 4.0 * 128 * 96 * args.pairs * (1024 * 1025 / 2)
+        line = {"metric": METRIC, "impl": "reference", "value": value, "unit": "TFLOP/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": 1e3 * step_flops / (value * 1e12), "higher_is_better": True,
+                "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": config_for(args),
+                "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                                 "sample": desc},
+                "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
     if args.config == "topk":
         vals, desc = [], ""
         for i in range(args.warmup + args.steps):
@@ -439,7 +511,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="stack",
                     choices=["stack", "qkv", "mlp_up", "mlp_down", "mlp_swiglu", "gemv", "tiny",
-                             "topk"])
+                             "topk", "attention"])
     ap.add_argument("--topk-n", type=int, default=200000, help="scores for --config topk")
     ap.add_argument("--topk-k", type=int, default=1000, help="k for --config topk")
     ap.add_argument("--m", type=int, default=32, help="tokens for --config gemv")
@@ -470,6 +542,10 @@ def main():
     elif args.config == "topk":
         wl = TopkWorkload(args.topk_n, args.topk_k, 5)
         unit = "GB/s"
+        units_per_step = None
+    elif args.config == "attention":
+        wl = AttentionWorkload(args.pairs, 1024, 96, 32768, 9)
+        unit = "TFLOP/s"
         units_per_step = None
     else:
         from paper_2608_30877_gb300 import synthetic as S
@@ -546,6 +622,10 @@ def main():
         if args.config == "topk":
             gbs, desc = oracle_topk_sample(args.topk_n, args.topk_k)
             line["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                    "sample": desc}
+        elif args.config == "attention":
+            tf, desc = oracle_attention_sample()
+            line["cpu_baseline"] = {"value": tf, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
                                     "sample": desc}
         elif args.config == "stack":
             mac_s, desc, threads = oracle_sample(S.D_MODEL, 2048, 15.0)

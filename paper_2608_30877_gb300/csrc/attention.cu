@@ -19,9 +19,11 @@
 //                shared memory as an MN-major operand (V is stored token-
 //                major, d contiguous -- exactly the layout the TMA box has);
 //   epilogue     O / l, bf16, 16-byte stores.
-// The MMA warp issues S of the next key block as soon as the softmax warps
-// have read S, so the softmax of block j+1 overlaps the PV product of block
-// j.  K/V blocks stream through a two-stage TMA ring.
+// S is double-buffered in tensor memory, so the MMA warp keeps the S product
+// of the block after next queued while the softmax warps work on one block;
+// K/V blocks stream through a three-stage TMA ring.  The softmax rolls over
+// 32-key chunks (two reads of S: max, then exponentials), skips the mask on
+// blocks every query sees in full, and raises its running max lazily.
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, waits for its own copies and MMAs and frees tensor memory.
 #include "internal.h"
@@ -36,7 +38,7 @@ namespace {
 constexpr int kD = 128;        // head dimension
 constexpr int kBQ = 128;       // queries per CTA (MMA M)
 constexpr int kBKV = 128;      // keys per block (MMA N of S, K of PV)
-constexpr int kKVStages = 2;
+constexpr int kKVStages = 3;
 constexpr int kThreads = 6 * 32;  // TMA warp, MMA warp, 4 softmax warps
 
 struct AttnLayout {
@@ -46,12 +48,13 @@ struct AttnLayout {
     static constexpr int K_OFF = Q_OFF + TILE;
     static constexpr int V_OFF = K_OFF + kKVStages * TILE;
     static constexpr int BAR_OFF = V_OFF + kKVStages * TILE;
-    // q_full, kv_full[S], kv_empty[S], s_full, s_free, p_full, o_ready, drain
-    static constexpr int NBARS = 1 + 2 * kKVStages + 5;
+    // q_full, kv_full[S], kv_empty[S], s_full[2], s_free[2], p_full, o_ready, drain
+    static constexpr int NBARS = 1 + 2 * kKVStages + 7;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
-    // tensor memory columns
-    static constexpr int S_COL = 0, P_COL = 128, O_COL = 256, TMEM_COLS = 512;
+    // tensor memory columns: two S buffers (blocks alternate), P, O
+    static constexpr int S_COL = 0, P_COL = 256, O_COL = 384, TMEM_COLS = 512;
+    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
 };
 
 // SS MMA: D[tmem] (+)= A[smem] * B[smem]^T, kind::f16.
@@ -78,6 +81,17 @@ __device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr, uint32_t
     d |= static_cast<uint64_t>(1) << 46;
     d |= static_cast<uint64_t>(2) << 61;
     return d;
+}
+
+// 32 lanes x 16 columns of 32 bits (see tmem_st_32x32b_x32).
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15])
+        : "memory");
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -166,11 +180,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t q_full = bars;
     auto kv_full = [&](int s) { return bars + 8u * (1 + s); };
     auto kv_empty = [&](int s) { return bars + 8u * (1 + kKVStages + s); };
-    const uint32_t s_full = bars + 8u * (1 + 2 * kKVStages);
-    const uint32_t s_free = s_full + 8u;
-    const uint32_t p_full = s_full + 16u;
-    const uint32_t o_ready = s_full + 24u;
-    const uint32_t drain = s_full + 32u;
+    auto s_full = [&](int b) { return bars + 8u * (1 + 2 * kKVStages + b); };
+    auto s_free = [&](int b) { return bars + 8u * (3 + 2 * kKVStages + b); };
+    const uint32_t p_full = bars + 8u * (5 + 2 * kKVStages);
+    const uint32_t o_ready = p_full + 8u;
+    const uint32_t drain = p_full + 16u;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
 
@@ -180,8 +194,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(kv_full(s), 1);
             mbar_init(kv_empty(s), 1);
         }
-        mbar_init(s_full, 1);
-        mbar_init(s_free, 4);   // one arrival per softmax warp
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(s_full(b), 1);
+            mbar_init(s_free(b), 4);  // one arrival per softmax warp
+        }
         mbar_init(p_full, 4);
         mbar_init(o_ready, 1);
         mbar_init(drain, 1);
@@ -243,28 +259,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
             constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
             bool ok = wait_one(q_full, 0, abort_flag, p.status);
+            // S of block j into buffer j & 1; that buffer's previous block is
+            // j - 2, read by the softmax warps before they free it
             auto issue_s = [&](int j) -> bool {
-                const int s = j % kKVStages;
+                const int s = j % kKVStages, b = j & 1;
                 if (!wait_one(kv_full(s), (j / kKVStages) & 1u, abort_flag, p.status)) return false;
-                // S may be overwritten once the softmax warps have read block j-1
-                if (j > 0 && !wait_one(s_free, (j - 1) & 1u, abort_flag, p.status)) return false;
+                if (j >= 2 && !wait_one(s_free(b), ((j - 2) >> 1) & 1u, abort_flag, p.status))
+                    return false;
                 tc_fence_after();
                 const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + s * L::TILE;
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
-                    tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
+                    tc_mma_ss(tmem + L::S_COL + b * kBKV, sdesc_kmajor_sw128(qs + off),
                               sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
                 }
-                tc_commit(s_full);
+                tc_commit(s_full(b));
                 return true;
             };
             if (ok && nblk > 0) ok = issue_s(0);
+            if (ok && nblk > 1) ok = issue_s(1);
             for (int j = 0; ok && j < nblk; ++j) {
-                if (j + 1 < nblk && !issue_s(j + 1)) {
-                    ok = false;
-                    break;
-                }
                 // O += P V once the softmax warps have written P of block j
                 if (!wait_one(p_full, j & 1u, abort_flag, p.status)) {
                     ok = false;
@@ -282,6 +297,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_commit(o_ready);
                 tc_commit(kv_empty(s));
+                if (j + 2 < nblk && !issue_s(j + 2)) {
+                    ok = false;
+                    break;
+                }
             }
             tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
             const uint64_t t0 = global_timer_ns();
@@ -296,49 +315,39 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = q0 + r;                   // query token
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const float c = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
+        // Running max m (log2 units, scale folded in) and sum l.  The max is
+        // raised lazily: only when a block's max exceeds it by more than 8
+        // (p <= 2^8 otherwise), so O is rescaled rarely; O and l always use
+        // the same m, so the final O / l is exact either way.
         float m = kMaskedScore, l = 0.0f;
         bool ok = true;
         for (int j = 0; ok && j < nblk; ++j) {
-            if (!wait_warp(s_full, j & 1u, abort_flag, p.status)) {
+            const int b = j & 1;
+            if (!wait_warp(s_full(b), (j >> 1) & 1u, abort_flag, p.status)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             const int kbase = ss + (b_first + j) * kBKV;
-            float sv[kBKV];
-#pragma unroll
+            // every key of the block allowed for every query of the block
+            const bool interior = kbase + kBKV - 1 <= q0 && kbase > q0 + kBQ - 1 - W;
+            const uint32_t s_tm = lane_base + L::S_COL + b * kBKV;
+            auto scaled = [&](uint32_t raw_bits, int key) -> float {
+                const bool allowed = interior || (key <= i && key > i - W && key < se);
+                return allowed ? __uint_as_float(raw_bits) * c : kMaskedScore;
+            };
+            float mb = kMaskedScore;
+#pragma unroll 1
             for (int ch = 0; ch < kBKV / 32; ++ch) {
                 uint32_t v[32];
-                tmem_ld_32x32b_x32(lane_base + L::S_COL + ch * 32, v);
+                tmem_ld_32x32b_x32(s_tm + ch * 32, v);
                 tmem_ld_wait(v);
 #pragma unroll
-                for (int t = 0; t < 32; ++t) {
-                    const int key = kbase + ch * 32 + t;
-                    const bool allowed = key <= i && key > i - W && key < se;
-                    sv[ch * 32 + t] = allowed ? __uint_as_float(v[t]) * c : kMaskedScore;
-                }
+                for (int t = 0; t < 32; ++t) mb = fmaxf(mb, scaled(v[t], kbase + ch * 32 + t));
             }
-            // S is in registers: the next block's S MMA may start
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(s_free);
-            float mb = kMaskedScore;
-#pragma unroll
-            for (int t = 0; t < kBKV; ++t) mb = fmaxf(mb, sv[t]);
-            const float m_new = fmaxf(m, mb);
+            const bool raise = mb > m + 8.0f;
+            const float m_new = raise ? mb : m;
             const float alpha = ex2(m - m_new);
-            float sum = 0.0f;
-            uint32_t pk[kBKV / 2];
-#pragma unroll
-            for (int t = 0; t < kBKV / 2; ++t) {
-                // masked keys get exactly 0 (a row may have none allowed in a block)
-                const float p0 = sv[2 * t] > kMaskedScore ? ex2(sv[2 * t] - m_new) : 0.0f;
-                const float p1 = sv[2 * t + 1] > kMaskedScore ? ex2(sv[2 * t + 1] - m_new) : 0.0f;
-                sum += p0 + p1;
-                pk[t] = pack_bf16x2_rn(p0, p1);
-            }
-            l = l * alpha + sum;
-            m = m_new;
             // P and O of block j-1 are in use until its PV product completes
             if (j > 0) {
                 if (!wait_warp(o_ready, (j - 1) & 1u, abort_flag, p.status)) {
@@ -346,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, alpha < 1.0f)) {
+                if (__any_sync(0xffffffffu, raise)) {
 #pragma unroll 1
                     for (int ch = 0; ch < kD / 32; ++ch) {
                         uint32_t v[32];
@@ -359,17 +368,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            uint32_t half[32];
+            l *= alpha;
+            m = m_new;
+            float sum = 0.0f;
+#pragma unroll 1
+            for (int ch = 0; ch < kBKV / 32; ++ch) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(s_tm + ch * 32, v);
+                tmem_ld_wait(v);
+                uint32_t pk[16];
 #pragma unroll
-            for (int t = 0; t < 32; ++t) half[t] = pk[t];
-            tmem_st_32x32b_x32(lane_base + L::P_COL, half);
-#pragma unroll
-            for (int t = 0; t < 32; ++t) half[t] = pk[32 + t];
-            tmem_st_32x32b_x32(lane_base + L::P_COL + 32, half);
+                for (int t = 0; t < 16; ++t) {
+                    // masked keys get exactly 0 (a row may have none allowed in a block)
+                    const float s0 = scaled(v[2 * t], kbase + ch * 32 + 2 * t);
+                    const float s1 = scaled(v[2 * t + 1], kbase + ch * 32 + 2 * t + 1);
+                    const float p0 = s0 > kMaskedScore ? ex2(s0 - m) : 0.0f;
+                    const float p1 = s1 > kMaskedScore ? ex2(s1 - m) : 0.0f;
+                    sum += p0 + p1;
+                    pk[t] = pack_bf16x2_rn(p0, p1);
+                }
+                tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
+            }
+            l += sum;
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(p_full);
+            if (lane == 0) {
+                mbar_arrive(s_free(b));  // S buffer b read in full
+                mbar_arrive(p_full);     // P of block j written
+            }
         }
         // ---- epilogue: O / l -> bf16
         if (ok && nblk > 0 && wait_warp(o_ready, (nblk - 1) & 1u, abort_flag, p.status)) {
