@@ -198,7 +198,7 @@ def make_weights(N, K, g, seed):
 
 
 class StackWorkload:
-    def __init__(self, pairs, tokens, layers, g=128):
+    def __init__(self, pairs, tokens, layers, g=128, graph=False):
         import torch
         from paper_2608_30877_gb300 import synthetic as S
         from paper_2608_30877_gb300 import w4a16 as W
@@ -225,10 +225,15 @@ class StackWorkload:
         self.entries = entries
         self.arr = W.make_layer_array(entries)
         self.launches_per_step = len(entries)
+        # one CUDA graph of the whole pass, replayed per step (w4a16_stack_graph_*)
+        self.graph = W.StackGraph(entries, self.M, g) if graph else None
 
     def step(self, stream=None):
         from paper_2608_30877_gb300 import w4a16 as W
-        W.linear_stack_array(self.arr, self.M, self.g, stream)
+        if self.graph is not None:
+            self.graph.launch(stream)
+        else:
+            W.linear_stack_array(self.arr, self.M, self.g, stream)
 
     def per_linear(self, reps=3):
         """Event-timed TFLOP/s of each linear shape (layer 0), outside the timed region."""
@@ -404,8 +409,10 @@ def config_for(args):
     if c == "stack":
         return {"workload": "175B-class int4 linear stack, 96 layers x {qkv 12288->36864, "
                             "o 12288->12288, up 12288->49152, down 49152->12288}, "
-                            f"M={args.pairs * 1024} ({args.pairs} pairs x 1024 tokens), g=128",
-                "pairs": args.pairs, "tokens_per_pair": 1024, "layers": args.layers, "g": 128,
+                            f"M={args.pairs * args.tokens} ({args.pairs} pairs x {args.tokens} tokens), "
+                            "g=128" + (", replayed as one CUDA graph" if args.graph else ""),
+                "pairs": args.pairs, "tokens_per_pair": args.tokens, "layers": args.layers, "g": 128,
+                "graph": bool(args.graph),
                 "l2": "inputs larger than L2 (88 GB packed weights, >=1.6 GB activations per "
                       "linear); no flush"}
     if c == "attention":
@@ -477,7 +484,7 @@ def run_reference(args):
     if args.config == "stack":
         K, N_rows = S.D_MODEL, 2048
         unit = "pairs/s"
-        per_unit = stack_macs_per_pair(1024, args.layers)
+        per_unit = stack_macs_per_pair(args.tokens, args.layers)
     else:
         cfg = config_for(args)
         K, N_rows = cfg["K"], min(cfg["N"], 2048)
@@ -516,6 +523,9 @@ def main():
     ap.add_argument("--topk-k", type=int, default=1000, help="k for --config topk")
     ap.add_argument("--m", type=int, default=32, help="tokens for --config gemv")
     ap.add_argument("--pairs", type=int, default=64)
+    ap.add_argument("--tokens", type=int, default=1024, help="tokens per pair for the stack")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay the stack as one captured CUDA graph")
     ap.add_argument("--layers", type=int, default=96)
     ap.add_argument("--ref-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -536,7 +546,7 @@ def main():
 
     setup_t0 = time.perf_counter()
     if args.config == "stack":
-        wl = StackWorkload(args.pairs, 1024, args.layers)
+        wl = StackWorkload(args.pairs, args.tokens, args.layers, graph=args.graph)
         unit = "pairs/s"
         units_per_step = wl.pairs
     elif args.config == "topk":
@@ -629,7 +639,7 @@ def main():
                                     "sample": desc}
         elif args.config == "stack":
             mac_s, desc, threads = oracle_sample(S.D_MODEL, 2048, 15.0)
-            cb = mac_s / stack_macs_per_pair(1024, args.layers)
+            cb = mac_s / stack_macs_per_pair(args.tokens, args.layers)
             line["cpu_baseline"] = {"value": cb, "unit": "pairs/s", "cores": threads,
                                     "kind": "oracle", "sample": desc}
         else:

@@ -135,6 +135,26 @@ int w4a16_linear_stack(const w4a16_layer* layers, int64_t n_layers,
                        int64_t M, int64_t g, void* stream);
 
 /*
+ * A layer stack captured once as a CUDA graph and replayed per batch: the
+ * continuous-batching loop of the paper's pipeline (Sec. 3.3) runs the same
+ * stack over batch after batch, with each batch's inputs copied into the same
+ * buffers.  Replaying the graph removes the per-layer host launch work.
+ *
+ * w4a16_stack_graph_create validates every layer (as w4a16_linear_stack) and
+ * captures the stack's launches -- the pointers in `layers` are baked in --
+ * into *out.  Unlike the per-call entry points it allocates: the graph and
+ * its host handle, released by w4a16_stack_graph_destroy.
+ * w4a16_stack_graph_launch enqueues one pass on `stream` (the current device
+ * must be the one the graph was created on, else W4A16_ERR_INVALID_ARG) and
+ * allocates nothing.  Results are bit-identical to w4a16_linear_stack.
+ */
+typedef struct w4a16_stack_graph w4a16_stack_graph;
+int w4a16_stack_graph_create(const w4a16_layer* layers, int64_t n_layers, int64_t M, int64_t g,
+                             w4a16_stack_graph** out);
+int w4a16_stack_graph_launch(w4a16_stack_graph* graph, void* stream);
+int w4a16_stack_graph_destroy(w4a16_stack_graph* graph);
+
+/*
  * wd = dequant(w_packed, scales) as bf16 [N, K] (device).  The same unpack
  * and rounding as inside the GEMM, exported so that it can be compared bit
  * for bit with the definition above.

@@ -11,6 +11,7 @@
 #include <cmath>
 #include <cstdlib>
 #include <mutex>
+#include <new>
 
 namespace w4a16 {
 namespace {
@@ -292,6 +293,77 @@ extern "C" int w4a16_linear_stack(const w4a16_layer* layers, int64_t n_layers, i
         if (rc != W4A16_OK) return rc;
     }
     return W4A16_OK;
+}
+
+// A captured layer stack: one CUDA graph of the stack's kernel launches.
+struct w4a16_stack_graph {
+    cudaGraphExec_t exec = nullptr;
+    int device = 0;
+};
+
+extern "C" int w4a16_stack_graph_create(const w4a16_layer* layers, int64_t n_layers, int64_t M,
+                                        int64_t g, w4a16_stack_graph** out) {
+    if (out == nullptr) return W4A16_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (layers == nullptr || n_layers <= 0) return W4A16_ERR_INVALID_ARG;
+    for (int64_t i = 0; i < n_layers; ++i) {
+        const w4a16_layer& l = layers[i];
+        const int rc = check_linear(l.x, l.w_packed, l.scales, l.out, M, l.N, l.K, g);
+        if (rc != W4A16_OK) return rc;
+    }
+    DeviceState* st = nullptr;
+    int rc = device_state(&st);
+    if (rc != W4A16_OK) return rc;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return W4A16_ERR_CUDA;
+    cudaStream_t cs = nullptr;
+    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return W4A16_ERR_CUDA;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    rc = W4A16_OK;
+    if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+        rc = W4A16_ERR_CUDA;
+    } else {
+        for (int64_t i = 0; i < n_layers && rc == W4A16_OK; ++i) {
+            const w4a16_layer& l = layers[i];
+            rc = launch_linear(*st, l.x, l.w_packed, l.scales, l.out, M, l.N, l.K, g,
+                               plain_epilogue(l.N), cs);
+        }
+        const cudaError_t e = cudaStreamEndCapture(cs, &graph);
+        if (rc == W4A16_OK && e != cudaSuccess) rc = W4A16_ERR_CUDA;
+    }
+    if (rc == W4A16_OK && cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) rc = W4A16_ERR_CUDA;
+    if (graph != nullptr) cudaGraphDestroy(graph);
+    cudaStreamDestroy(cs);
+    if (rc != W4A16_OK) {
+        if (exec != nullptr) cudaGraphExecDestroy(exec);
+        return rc;
+    }
+    w4a16_stack_graph* h = new (std::nothrow) w4a16_stack_graph;
+    if (h == nullptr) {
+        cudaGraphExecDestroy(exec);
+        return W4A16_ERR_CUDA;
+    }
+    h->exec = exec;
+    h->device = dev;
+    *out = h;
+    return W4A16_OK;
+}
+
+extern "C" int w4a16_stack_graph_launch(w4a16_stack_graph* graph, void* stream) {
+    if (graph == nullptr || graph->exec == nullptr) return W4A16_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev != graph->device) return W4A16_ERR_INVALID_ARG;
+    return cudaGraphLaunch(graph->exec, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? W4A16_OK
+               : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_stack_graph_destroy(w4a16_stack_graph* graph) {
+    if (graph == nullptr) return W4A16_ERR_INVALID_ARG;
+    const cudaError_t e = graph->exec != nullptr ? cudaGraphExecDestroy(graph->exec) : cudaSuccess;
+    delete graph;
+    return e == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
 extern "C" int w4a16_dequant(const void* w_packed_u8, const void* scales_bf16, void* w_bf16,

@@ -53,6 +53,10 @@ def lib() -> ctypes.CDLL:
         L.w4a16_linear_fused.argtypes = [p, p, p, p, p, p, i64, i64, i64, i64, ctypes.c_int, p]
         L.w4a16_linear_stack.argtypes = [ctypes.POINTER(Layer), i64, i64, i64, p]
         L.w4a16_dequant.argtypes = [p, p, p, i64, i64, i64, p]
+        L.w4a16_stack_graph_create.argtypes = [ctypes.POINTER(Layer), i64, i64, i64,
+                                               ctypes.POINTER(ctypes.c_void_p)]
+        L.w4a16_stack_graph_launch.argtypes = [p, p]
+        L.w4a16_stack_graph_destroy.argtypes = [p]
         L.w4a16_gather_rows.argtypes = [p, i64, i64, p, i64, p, p]
         L.w4a16_attention_prefill.argtypes = [p, p, i64, i64, i64, i64, i64, p, p]
         L.w4a16_topk_smallest.argtypes = [p, ctypes.c_int, i64, i64, p, p, p]
@@ -63,7 +67,9 @@ def lib() -> ctypes.CDLL:
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
         for f in ("w4a16_linear", "w4a16_linear_fused", "w4a16_linear_stack",
-                  "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_attention_prefill", "w4a16_dequant", "w4a16_quantize",
+                  "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_attention_prefill",
+                  "w4a16_stack_graph_create", "w4a16_stack_graph_launch",
+                  "w4a16_stack_graph_destroy", "w4a16_dequant", "w4a16_quantize",
                   "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
@@ -154,6 +160,31 @@ def make_layer_array(layers) -> ctypes.Array:
         arr[i] = Layer(x.data_ptr(), w.data_ptr(), s.data_ptr(), o.data_ptr(), w.shape[0],
                        w.shape[1] * 2)
     return arr
+
+
+class StackGraph:
+    """A layer stack captured as a CUDA graph (include/w4a16.h); replay with
+    launch(), release with close() (or as a context manager)."""
+
+    def __init__(self, layers, M: int, g: int = 128):
+        self._arr = make_layer_array(layers)
+        self._h = ctypes.c_void_p()
+        _check("w4a16_stack_graph_create", lib().w4a16_stack_graph_create(
+            self._arr, len(self._arr), M, g, ctypes.byref(self._h)))
+
+    def launch(self, stream=None):
+        _check("w4a16_stack_graph_launch", lib().w4a16_stack_graph_launch(self._h, _stream(stream)))
+
+    def close(self):
+        if self._h:
+            _check("w4a16_stack_graph_destroy", lib().w4a16_stack_graph_destroy(self._h))
+            self._h = ctypes.c_void_p()
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
 
 
 def linear_stack_array(arr: ctypes.Array, M: int, g: int = 128, stream=None) -> None:

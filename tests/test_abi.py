@@ -103,3 +103,17 @@ def test_attention_rejects_before_launch(L):
     assert L.w4a16_attention_prefill(A, 2 * A, 1, 64, 2, 128, 0, 3 * A, None) == W.ERR_INVALID_ARG
     assert L.w4a16_attention_prefill(A, 2 * A + 4, 1, 64, 2, 128, 9, 3 * A, None) == W.ERR_ALIGNMENT
     assert L.w4a16_attention_prefill(A, 2 * A, 1, 64, 2, 128, 9, A + 64, None) == W.ERR_INVALID_ARG
+
+
+def test_stack_graph_rejects_bad_handles(L):
+    import ctypes
+    h = ctypes.c_void_p()
+    good = W.Layer(A, 2 * A, 3 * A, 4 * A, 8, 256)
+    arr = (W.Layer * 1)(good)
+    assert L.w4a16_stack_graph_create(arr, 1, 4, 128, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_stack_graph_create(None, 1, 4, 128, ctypes.byref(h)) == W.ERR_INVALID_ARG
+    bad = (W.Layer * 1)(W.Layer(A, 2 * A, 3 * A, 4 * A, 8, 200))
+    assert L.w4a16_stack_graph_create(bad, 1, 4, 128, ctypes.byref(h)) == W.ERR_INVALID_ARG
+    assert not h.value
+    assert L.w4a16_stack_graph_launch(None, None) == W.ERR_INVALID_ARG
+    assert L.w4a16_stack_graph_destroy(None) == W.ERR_INVALID_ARG
