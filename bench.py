@@ -151,29 +151,47 @@ def dist_env():
     return world, rank, local
 
 
-def init_dist(world, local):
+def init_dist(world, local, backend="nccl"):
+    """One process per GPU (nccl); gloo runs the same host logic on CPU."""
     import torch
     import torch.distributed as dist
     if world > 1 and not dist.is_initialized():
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
     return dist if world > 1 else None
+
+
+def _cuda_ok():
+    import torch
+    return torch.cuda.is_available()
 
 
 def barrier(dist):
     import torch
     if dist is not None:
         dist.barrier()
-    torch.cuda.synchronize()
+    if _cuda_ok():
+        torch.cuda.synchronize()
 
 
 def max_over_ranks(dist, v: float) -> float:
+    """The slowest rank's time: the job is done when every replica is."""
     import torch
     if dist is None:
         return v
-    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def replica_value(world: int, units_per_step: float, step_s: float) -> float:
+    """Whole-job throughput of N replicas (weak scaling): every rank runs the
+    same per-GPU work, so units of all ranks over the slowest rank's time."""
+    return world * units_per_step / step_s
 
 
 # ----------------------------------------------------------------- workloads
@@ -589,7 +607,7 @@ def main():
         raise RuntimeError("device status word set during the timed region")
 
     if args.config == "stack":
-        value = world * units_per_step / step_s
+        value = replica_value(world, units_per_step, step_s)
     elif args.config in ("gemv", "topk"):
         value = world * wl.bytes / step_s / 1e9
     else:
