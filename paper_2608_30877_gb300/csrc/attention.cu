@@ -19,9 +19,10 @@
 //                shared memory as an MN-major operand (V is stored token-
 //                major, d contiguous -- exactly the layout the TMA box has);
 //   epilogue     O / l, bf16, 16-byte stores.
-// S is double-buffered in tensor memory, so the MMA warp keeps the S product
-// of the block after next queued while the softmax warps work on one block;
-// K/V blocks stream through a three-stage TMA ring.  The softmax rolls over
+// Two CTAs share an SM (256 tensor-memory columns, 96 KB of shared memory),
+// so one CTA's loads, setup and epilogue overlap the other's MMAs: S of a
+// block is written into the columns P of the previous block used, once its
+// PV product is done, and K/V arrive one block at a time.  The softmax rolls over
 // 32-key chunks (two reads of S: max, then exponentials), skips the mask on
 // blocks every query sees in full, and raises its running max lazily.
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
@@ -38,7 +39,6 @@ namespace {
 constexpr int kD = 128;        // head dimension
 constexpr int kBQ = 128;       // queries per CTA (MMA M)
 constexpr int kBKV = 128;      // keys per block (MMA N of S, K of PV)
-constexpr int kKVStages = 3;
 constexpr int kThreads = 6 * 32;  // TMA warp, MMA warp, 4 softmax warps
 
 struct AttnLayout {
@@ -46,14 +46,15 @@ struct AttnLayout {
     static constexpr int TILE = 2 * BOX;           // [128 x 128]: 32 KB
     static constexpr int Q_OFF = 0;
     static constexpr int K_OFF = Q_OFF + TILE;
-    static constexpr int V_OFF = K_OFF + kKVStages * TILE;
-    static constexpr int BAR_OFF = V_OFF + kKVStages * TILE;
-    // q_full, kv_full[S], kv_empty[S], s_full[2], s_free[2], p_full, o_ready, drain
-    static constexpr int NBARS = 1 + 2 * kKVStages + 7;
+    static constexpr int V_OFF = K_OFF + TILE;
+    static constexpr int BAR_OFF = V_OFF + TILE;
+    // q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, o_ready, drain
+    static constexpr int NBARS = 9;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
-    // tensor memory columns: two S buffers (blocks alternate), P, O
-    static constexpr int S_COL = 0, P_COL = 256, O_COL = 384, TMEM_COLS = 512;
+    // tensor memory columns: S, with P written over it in place, and O; 256
+    // columns and under 113 KB of shared memory let two CTAs share an SM
+    static constexpr int S_COL = 0, P_COL = 0, O_COL = 128, TMEM_COLS = 256;
     static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
 };
 
@@ -108,7 +109,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
 
 constexpr float kMaskedScore = -1.0e30f;  // finite: fully masked rows stay NaN-free
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p) {
     using L = AttnLayout;
     extern __shared__ uint8_t smem_raw[];
@@ -178,27 +179,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const uint32_t bars = sbase + L::BAR_OFF;
     const uint32_t q_full = bars;
-    auto kv_full = [&](int s) { return bars + 8u * (1 + s); };
-    auto kv_empty = [&](int s) { return bars + 8u * (1 + kKVStages + s); };
-    auto s_full = [&](int b) { return bars + 8u * (1 + 2 * kKVStages + b); };
-    auto s_free = [&](int b) { return bars + 8u * (3 + 2 * kKVStages + b); };
-    const uint32_t p_full = bars + 8u * (5 + 2 * kKVStages);
-    const uint32_t o_ready = p_full + 8u;
-    const uint32_t drain = p_full + 16u;
+    const uint32_t k_full = bars + 8u, k_empty = bars + 16u;
+    const uint32_t v_full = bars + 24u, v_empty = bars + 32u;
+    const uint32_t s_full = bars + 40u, p_full = bars + 48u;
+    const uint32_t o_ready = bars + 56u, drain = bars + 64u;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
-        for (int s = 0; s < kKVStages; ++s) {
-            mbar_init(kv_full(s), 1);
-            mbar_init(kv_empty(s), 1);
-        }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(s_full(b), 1);
-            mbar_init(s_free(b), 4);  // one arrival per softmax warp
-        }
-        mbar_init(p_full, 4);
+        mbar_init(k_full, 1);
+        mbar_init(k_empty, 1);
+        mbar_init(v_full, 1);
+        mbar_init(v_empty, 1);
+        mbar_init(s_full, 1);
+        mbar_init(p_full, 4);  // one arrival per softmax warp
         mbar_init(o_ready, 1);
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -222,36 +217,38 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(q_full, L::TILE);
             tma_load_2d(sbase + L::Q_OFF, &tmap_qkv, q_full, h * kD, q0);
             tma_load_2d(sbase + L::Q_OFF + L::BOX, &tmap_qkv, q_full, h * kD + 64, q0);
-            int j = 0;
-            for (; ok && j < nblk; ++j) {
-                const int s = j % kKVStages;
-                if (!wait_one(kv_empty(s), ((j / kKVStages) & 1u) ^ 1u, abort_flag, p.status)) {
+            // K of a block is free once its S product is done, V once its PV
+            // product is: K of block j + 1 loads while block j's softmax runs
+            int nk = 0, nv = 0;
+            for (int j = 0; ok && j < nblk; ++j) {
+                const int row = ss + (b_first + j) * kBKV;
+                if (!wait_one(k_empty, (j & 1u) ^ 1u, abort_flag, p.status)) {
                     ok = false;
                     break;
                 }
-                const int row = ss + (b_first + j) * kBKV;
-                mbar_arrive_expect_tx(kv_full(s), 2 * L::TILE);
-                const uint32_t ks = sbase + L::K_OFF + s * L::TILE;
-                const uint32_t vs = sbase + L::V_OFF + s * L::TILE;
-                tma_load_2d(ks, &tmap_qkv, kv_full(s), Hd + h * kD, row);
-                tma_load_2d(ks + L::BOX, &tmap_qkv, kv_full(s), Hd + h * kD + 64, row);
-                tma_load_2d(vs, &tmap_qkv, kv_full(s), 2 * Hd + h * kD, row);
-                tma_load_2d(vs + L::BOX, &tmap_qkv, kv_full(s), 2 * Hd + h * kD + 64, row);
+                mbar_arrive_expect_tx(k_full, L::TILE);
+                tma_load_2d(sbase + L::K_OFF, &tmap_qkv, k_full, Hd + h * kD, row);
+                tma_load_2d(sbase + L::K_OFF + L::BOX, &tmap_qkv, k_full, Hd + h * kD + 64, row);
+                ++nk;
+                if (!wait_one(v_empty, (j & 1u) ^ 1u, abort_flag, p.status)) {
+                    ok = false;
+                    break;
+                }
+                mbar_arrive_expect_tx(v_full, L::TILE);
+                tma_load_2d(sbase + L::V_OFF, &tmap_qkv, v_full, 2 * Hd + h * kD, row);
+                tma_load_2d(sbase + L::V_OFF + L::BOX, &tmap_qkv, v_full, 2 * Hd + h * kD + 64, row);
+                ++nv;
             }
             // every load issued has landed before exit
-            {
+            auto settle = [&](uint32_t bar, uint32_t parity) {
                 const uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(q_full, 0)) {
+                while (!mbar_try_wait(bar, parity)) {
                     if (global_timer_ns() - t0 > kWaitLimitNs) break;
                 }
-            }
-            const int last = j < kKVStages ? j : kKVStages;
-            for (int i = j - last; i < j; ++i) {
-                const uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(kv_full(i % kKVStages), (i / kKVStages) & 1u)) {
-                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
-                }
-            }
+            };
+            settle(q_full, 0);
+            if (nk > 0) settle(k_full, (nk - 1) & 1u);
+            if (nv > 0) settle(v_full, (nv - 1) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -259,35 +256,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
             constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
             bool ok = wait_one(q_full, 0, abort_flag, p.status);
-            // S of block j into buffer j & 1; that buffer's previous block is
-            // j - 2, read by the softmax warps before they free it
+            // S of block j; P of block j - 1 lives in the same columns, so S
+            // waits for that block's PV product to complete
             auto issue_s = [&](int j) -> bool {
-                const int s = j % kKVStages, b = j & 1;
-                if (!wait_one(kv_full(s), (j / kKVStages) & 1u, abort_flag, p.status)) return false;
-                if (j >= 2 && !wait_one(s_free(b), ((j - 2) >> 1) & 1u, abort_flag, p.status))
-                    return false;
+                if (!wait_one(k_full, j & 1u, abort_flag, p.status)) return false;
+                if (j >= 1 && !wait_one(o_ready, (j - 1) & 1u, abort_flag, p.status)) return false;
                 tc_fence_after();
-                const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + s * L::TILE;
+                const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF;
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
-                    tc_mma_ss(tmem + L::S_COL + b * kBKV, sdesc_kmajor_sw128(qs + off),
+                    tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
                               sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
                 }
-                tc_commit(s_full(b));
+                tc_commit(s_full);
+                tc_commit(k_empty);
                 return true;
             };
             if (ok && nblk > 0) ok = issue_s(0);
-            if (ok && nblk > 1) ok = issue_s(1);
             for (int j = 0; ok && j < nblk; ++j) {
                 // O += P V once the softmax warps have written P of block j
-                if (!wait_one(p_full, j & 1u, abort_flag, p.status)) {
+                if (!wait_one(p_full, j & 1u, abort_flag, p.status) ||
+                    !wait_one(v_full, j & 1u, abort_flag, p.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const int s = j % kKVStages;
-                const uint32_t vs = sbase + L::V_OFF + s * L::TILE;
+                const uint32_t vs = sbase + L::V_OFF;
 #pragma unroll
                 for (int kk = 0; kk < kBKV / 16; ++kk) {
                     // keys 16 kk .. 16 kk + 15: rows of the V tile; P columns 8 kk ..
@@ -296,8 +291,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                               (j > 0 || kk > 0) ? 1u : 0u);
                 }
                 tc_commit(o_ready);
-                tc_commit(kv_empty(s));
-                if (j + 2 < nblk && !issue_s(j + 2)) {
+                tc_commit(v_empty);
+                if (j + 1 < nblk && !issue_s(j + 1)) {
                     ok = false;
                     break;
                 }
@@ -322,8 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float m = kMaskedScore, l = 0.0f;
         bool ok = true;
         for (int j = 0; ok && j < nblk; ++j) {
-            const int b = j & 1;
-            if (!wait_warp(s_full(b), (j >> 1) & 1u, abort_flag, p.status)) {
+            if (!wait_warp(s_full, j & 1u, abort_flag, p.status)) {
                 ok = false;
                 break;
             }
@@ -331,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int kbase = ss + (b_first + j) * kBKV;
             // every key of the block allowed for every query of the block
             const bool interior = kbase + kBKV - 1 <= q0 && kbase > q0 + kBQ - 1 - W;
-            const uint32_t s_tm = lane_base + L::S_COL + b * kBKV;
+            const uint32_t s_tm = lane_base + L::S_COL;
             auto scaled = [&](uint32_t raw_bits, int key) -> float {
                 const bool allowed = interior || (key <= i && key > i - W && key < se);
                 return allowed ? __uint_as_float(raw_bits) * c : kMaskedScore;
@@ -393,10 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(s_free(b));  // S buffer b read in full
-                mbar_arrive(p_full);     // P of block j written
-            }
+            if (lane == 0) mbar_arrive(p_full);  // P of block j written over S
         }
         // ---- epilogue: O / l -> bf16
         if (ok && nblk > 0 && wait_warp(o_ready, (nblk - 1) & 1u, abort_flag, p.status)) {
