@@ -107,7 +107,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
     return r;
 }
 
-constexpr float kMaskedScore = -1.0e30f;  // finite: fully masked rows stay NaN-free
+// Initial running max: finite, so 2^(s - m) of a masked (-inf) score is 0, never NaN.
+constexpr float kMaskedScore = -1.0e30f;
 
 __global__ void __launch_bounds__(kThreads, 2)
     attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p) {
@@ -326,23 +327,51 @@ __global__ void __launch_bounds__(kThreads, 2)
             // every key of the block allowed for every query of the block
             const bool interior = kbase + kBKV - 1 <= q0 && kbase > q0 + kBQ - 1 - W;
             const uint32_t s_tm = lane_base + L::S_COL;
-            auto scaled = [&](uint32_t raw_bits, int key) -> float {
-                const bool allowed = interior || (key <= i && key > i - W && key < se);
-                return allowed ? __uint_as_float(raw_bits) * c : kMaskedScore;
-            };
-            float mb = kMaskedScore;
-#pragma unroll 1
-            for (int ch = 0; ch < kBKV / 32; ++ch) {
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(s_tm + ch * 32, v);
-                tmem_ld_wait(v);
+            // the row's 128 raw scores, read once; masked keys become -inf, so
+            // their p = 2^(-inf) is exactly 0 with no compare in the exp loop
+            uint32_t v[kBKV / 32][32];
 #pragma unroll
-                for (int t = 0; t < 32; ++t) mb = fmaxf(mb, scaled(v[t], kbase + ch * 32 + t));
+            for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_32x32b_x32(s_tm + ch * 32, v[ch]);
+#pragma unroll
+            for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_wait(v[ch]);
+            if (!interior) {
+#pragma unroll
+                for (int ch = 0; ch < kBKV / 32; ++ch) {
+#pragma unroll
+                    for (int t = 0; t < 32; ++t) {
+                        const int key = kbase + ch * 32 + t;
+                        if (!(key <= i && key > i - W && key < se)) v[ch][t] = 0xFF800000u;
+                    }
+                }
             }
+            float mr[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int ch = 0; ch < kBKV / 32; ++ch) {
+#pragma unroll
+                for (int t = 0; t < 32; ++t) mr[t & 3] = fmaxf(mr[t & 3], __uint_as_float(v[ch][t]));
+            }
+            const float mb = fmaxf(fmaxf(mr[0], mr[1]), fmaxf(mr[2], mr[3])) * c;  // c > 0
             const bool raise = mb > m + 8.0f;
             const float m_new = raise ? mb : m;
             const float alpha = ex2(m - m_new);
-            // P and O of block j-1 are in use until its PV product completes
+            const float nm = -m_new;
+            float sum0 = 0.0f, sum1 = 0.0f;
+#pragma unroll
+            for (int ch = 0; ch < kBKV / 32; ++ch) {
+                uint32_t pk[16];
+#pragma unroll
+                for (int t = 0; t < 16; ++t) {
+                    const float p0 = ex2(fmaf(__uint_as_float(v[ch][2 * t]), c, nm));
+                    const float p1 = ex2(fmaf(__uint_as_float(v[ch][2 * t + 1]), c, nm));
+                    sum0 += p0;
+                    sum1 += p1;
+                    pk[t] = pack_bf16x2_rn(p0, p1);
+                }
+                tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
+            }
+            const float sum = sum0 + sum1;
+            // rescale O (the sum over blocks before j) to the new max; the PV
+            // product of block j-1 has completed, as S of block j followed it
             if (j > 0) {
                 if (!wait_warp(o_ready, (j - 1) & 1u, abort_flag, p.status)) {
                     ok = false;
@@ -352,38 +381,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                 if (__any_sync(0xffffffffu, raise)) {
 #pragma unroll 1
                     for (int ch = 0; ch < kD / 32; ++ch) {
-                        uint32_t v[32];
-                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
-                        tmem_ld_wait(v);
+                        uint32_t o[32];
+                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                        tmem_ld_wait(o);
 #pragma unroll
                         for (int t = 0; t < 32; ++t)
-                            v[t] = __float_as_uint(__uint_as_float(v[t]) * alpha);
-                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
+                            o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
+                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
                     }
                 }
             }
-            l *= alpha;
+            l = l * alpha + sum;
             m = m_new;
-            float sum = 0.0f;
-#pragma unroll 1
-            for (int ch = 0; ch < kBKV / 32; ++ch) {
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(s_tm + ch * 32, v);
-                tmem_ld_wait(v);
-                uint32_t pk[16];
-#pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    // masked keys get exactly 0 (a row may have none allowed in a block)
-                    const float s0 = scaled(v[2 * t], kbase + ch * 32 + 2 * t);
-                    const float s1 = scaled(v[2 * t + 1], kbase + ch * 32 + 2 * t + 1);
-                    const float p0 = s0 > kMaskedScore ? ex2(s0 - m) : 0.0f;
-                    const float p1 = s1 > kMaskedScore ? ex2(s1 - m) : 0.0f;
-                    sum += p0 + p1;
-                    pk[t] = pack_bf16x2_rn(p0, p1);
-                }
-                tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
-            }
-            l += sum;
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
