@@ -101,6 +101,40 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
+// max of three (a single instruction on sm_100 and later)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// (a.x b + c, a.y b + c) as one paired fp32 FMA, round to nearest
+__device__ __forceinline__ float2 ffma2(float2 a, float b, float c) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\t"
+        "mov.b64 rb, {%4, %4};\n\t"
+        "mov.b64 rc, {%5, %5};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\t"
+        "mov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b), "f"(c));
+    return d;
+}
+
+// paired fp32 add, round to nearest
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\t"
+        "mov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\t"
+        "mov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
@@ -334,42 +368,59 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_32x32b_x32(s_tm + ch * 32, v[ch]);
 #pragma unroll
             for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_wait(v[ch]);
-            if (!interior) {
+            // allowed key offsets in the block for query i: lo .. hi (keys past
+            // the end of the sequence only meet rows past it, never stored)
+            const int hi = i - kbase, lo = i - W + 1 - kbase;
+            // live[ch]: some lane of the warp has an allowed key in chunk ch
+            bool live[kBKV / 32];
 #pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) {
+            for (int ch = 0; ch < kBKV / 32; ++ch) {
+                live[ch] = interior || __any_sync(0xffffffffu, hi >= ch * 32 && lo <= ch * 32 + 31);
+                if (!interior && live[ch] &&
+                    __any_sync(0xffffffffu, hi < ch * 32 + 31 || lo > ch * 32)) {
 #pragma unroll
                     for (int t = 0; t < 32; ++t) {
-                        const int key = kbase + ch * 32 + t;
-                        if (!(key <= i && key > i - W && key < se)) v[ch][t] = 0xFF800000u;
+                        const int k = ch * 32 + t;
+                        if (k > hi || k < lo) v[ch][t] = 0xFF800000u;
                     }
                 }
             }
-            float mr[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
             for (int ch = 0; ch < kBKV / 32; ++ch) {
+                if (!live[ch]) continue;
 #pragma unroll
-                for (int t = 0; t < 32; ++t) mr[t & 3] = fmaxf(mr[t & 3], __uint_as_float(v[ch][t]));
+                for (int t = 0; t < 32; t += 4) {
+                    mx0 = fmax3(mx0, __uint_as_float(v[ch][t]), __uint_as_float(v[ch][t + 1]));
+                    mx1 = fmax3(mx1, __uint_as_float(v[ch][t + 2]), __uint_as_float(v[ch][t + 3]));
+                }
             }
-            const float mb = fmaxf(fmaxf(mr[0], mr[1]), fmaxf(mr[2], mr[3])) * c;  // c > 0
+            const float mb = fmaxf(mx0, mx1) * c;  // c > 0
             const bool raise = mb > m + 8.0f;
             const float m_new = raise ? mb : m;
             const float alpha = ex2(m - m_new);
             const float nm = -m_new;
-            float sum0 = 0.0f, sum1 = 0.0f;
+            float2 sum = make_float2(0.0f, 0.0f);
 #pragma unroll
             for (int ch = 0; ch < kBKV / 32; ++ch) {
                 uint32_t pk[16];
+                if (live[ch]) {
 #pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    const float p0 = ex2(fmaf(__uint_as_float(v[ch][2 * t]), c, nm));
-                    const float p1 = ex2(fmaf(__uint_as_float(v[ch][2 * t + 1]), c, nm));
-                    sum0 += p0;
-                    sum1 += p1;
-                    pk[t] = pack_bf16x2_rn(p0, p1);
+                    for (int t = 0; t < 16; ++t) {
+                        // p = 2^(s c - m) for a key pair: one paired FMA, two ex2
+                        float2 e = ffma2(make_float2(__uint_as_float(v[ch][2 * t]),
+                                                     __uint_as_float(v[ch][2 * t + 1])), c, nm);
+                        e.x = ex2(e.x);
+                        e.y = ex2(e.y);
+                        sum = fadd2(sum, e);
+                        pk[t] = pack_bf16x2_rn(e.x, e.y);
+                    }
+                } else {
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) pk[t] = 0u;
                 }
                 tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
             }
-            const float sum = sum0 + sum1;
             // rescale O (the sum over blocks before j) to the new max; the PV
             // product of block j-1 has completed, as S of block j followed it
             if (j > 0) {
@@ -391,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     }
                 }
             }
-            l = l * alpha + sum;
+            l = l * alpha + (sum.x + sum.y);
             m = m_new;
             tmem_st_wait();
             tc_fence_before();
