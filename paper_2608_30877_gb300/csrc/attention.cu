@@ -6,25 +6,26 @@
 //   o[i, h, :] = sum_j softmax_j(q_i . k_j / sqrt(d)) v_j,
 //   j in the sequence of i, i - W < j <= i;  d = 128.
 //
-// One CTA per (128-query block, head), flash-attention style on the
+// A job is one (128-query block, head), flash-attention style on the
 // 5th-generation tensor core:
 //   S  = Q K^T   tcgen05.mma kind::f16, A = Q and B = K from shared memory
 //                (TMA, 128-byte swizzle, K-major), S fp32 in tensor memory;
-//   softmax      four warps, thread = query row: tcgen05.ld of its S row,
-//                mask, running max and sum in fp32 (exp2 with the scale
-//                folded in), P as bf16 pairs written back into tensor memory
-//                with tcgen05.st; O rescaled in tensor memory when the
-//                running max grows;
+//   softmax      four warps, thread = query row: tcgen05.ld of its S row into
+//                registers, causal/window mask per 32-key chunk, running max
+//                and sum in fp32 (exp2 with the scale folded in), P as bf16
+//                pairs written over S with tcgen05.st; O rescaled in tensor
+//                memory when the running max grows (lazily, by more than 2^8);
 //   O += P V     tcgen05.mma with A = P from tensor memory and B = V from
 //                shared memory as an MN-major operand (V is stored token-
 //                major, d contiguous -- exactly the layout the TMA box has);
 //   epilogue     O / l, bf16, 16-byte stores.
-// Two CTAs share an SM (256 tensor-memory columns, 96 KB of shared memory),
-// so one CTA's loads, setup and epilogue overlap the other's MMAs: S of a
-// block is written into the columns P of the previous block used, once its
-// PV product is done, and K/V arrive one block at a time.  The softmax rolls over
-// 32-key chunks (two reads of S: max, then exponentials), skips the mask on
-// blocks every query sees in full, and raises its running max lazily.
+// The kernel is persistent with two CTAs per SM (256 tensor-memory columns
+// and 96 KB of shared memory each), every CTA taking every grid-th job, heads
+// fastest; one CTA's softmax and epilogue overlap the other's MMAs.  Within a
+// CTA the roles are one TMA warp, one MMA warp and the four softmax warps,
+// linked by mbarriers whose phases run on across jobs: Q and K of the next
+// job load during the current job's last softmax, and its first S product
+// runs during the current job's epilogue.
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, waits for its own copies and MMAs and frees tensor memory.
 #include "internal.h"
@@ -47,15 +48,20 @@ struct AttnLayout {
     static constexpr int Q_OFF = 0;
     static constexpr int K_OFF = Q_OFF + TILE;
     static constexpr int V_OFF = K_OFF + TILE;
-    static constexpr int BAR_OFF = V_OFF + TILE;
-    // q_full, k_full, k_empty, v_full, v_empty, s_full, p_full, o_ready, drain
-    static constexpr int NBARS = 9;
+    // epilogue staging: per softmax warp 32 rows x 32 columns of bf16 output
+    static constexpr int STAGE_OFF = V_OFF + TILE;
+    static constexpr int STAGE_WARP = 32 * 64;
+    static constexpr int BAR_OFF = STAGE_OFF + 4 * STAGE_WARP;
+    // q_full, q_empty, k_full, k_empty, v_full, v_empty, s_full, p_full,
+    // o_ready, drain
+    static constexpr int NBARS = 10;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
     // tensor memory columns: S, with P written over it in place, and O; 256
     // columns and under 113 KB of shared memory let two CTAs share an SM
     static constexpr int S_COL = 0, P_COL = 0, O_COL = 128, TMEM_COLS = 256;
-    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
+    // two CTAs per SM: 228 KB per SM, 1 KB of it reserved per CTA
+    static_assert(2 * (SMEM_BYTES + 1024) <= 228 * 1024, "shared memory");
 };
 
 // SS MMA: D[tmem] (+)= A[smem] * B[smem]^T, kind::f16.
@@ -144,8 +150,77 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
 // Initial running max: finite, so 2^(s - m) of a masked (-inf) score is 0, never NaN.
 constexpr float kMaskedScore = -1.0e30f;
 
+// One unit of work: query block [q0, q0 + 128) of the sequence [ss, se),
+// for head h.
+struct AttnJob {
+    int ss, se, q0, h;
+    bool valid;
+};
+
+// Resumable warp-collective search for the x-th query block over the
+// sequences (blocks of a sequence numbered from its last, the heaviest under
+// the causal mask, down).  x never decreases between calls of one warp, so
+// the search resumes at the 32-sequence group where the last one ended.
+struct JobCursor {
+    int s0 = 0;    // first sequence of the current group
+    int base = 0;  // query blocks of the sequences before s0
+};
+
+__device__ __forceinline__ bool find_block(const AttnParams& p, int x, int lane, JobCursor& cur,
+                                           int& ss, int& se, int& q0) {
+    for (; cur.s0 < p.nseq; cur.s0 += 32) {
+        const int s = cur.s0 + lane;
+        int a = 0, b = 0, nqb = 0;
+        if (s < p.nseq) {
+            a = p.seq_start[s];
+            b = p.seq_start[s + 1];
+            nqb = b > a ? (b - a + kBQ - 1) / kBQ : 0;
+        }
+        int incl = nqb;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
+        }
+        const int excl = incl - nqb;
+        const bool mine = s < p.nseq && x >= cur.base + excl && x < cur.base + incl;
+        const unsigned who = __ballot_sync(0xffffffffu, mine);
+        if (who) {
+            const int src = __ffs(who) - 1;
+            const int e = __shfl_sync(0xffffffffu, excl, src);
+            const int n = __shfl_sync(0xffffffffu, nqb, src);
+            ss = __shfl_sync(0xffffffffu, a, src);
+            se = __shfl_sync(0xffffffffu, b, src);
+            q0 = ss + (n - 1 - (x - cur.base - e)) * kBQ;
+            return true;
+        }
+        cur.base += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    return false;
+}
+
+// Job t of the CTA's sequence t = blockIdx.x, blockIdx.x + gridDim.x, ...:
+// heads vary fastest, so the CTAs running at one time share the K/V of a
+// few sequences in L2.
+__device__ __forceinline__ AttnJob job_at(const AttnParams& p, int64_t t, int lane, JobCursor& cur) {
+    AttnJob j{};
+    const int x = static_cast<int>(t / p.H);
+    j.h = static_cast<int>(t % p.H);
+    j.valid = find_block(p, x, lane, cur, j.ss, j.se, j.q0);
+    return j;
+}
+
+// key blocks of the sequence that some query of the block can see
+__device__ __forceinline__ void key_range(const AttnJob& jb, int W, int& b_first, int& nblk) {
+    const int q_last = (jb.q0 + kBQ - 1 < jb.se - 1 ? jb.q0 + kBQ - 1 : jb.se - 1);
+    const int k_first = jb.q0 - W + 1 > jb.ss ? jb.q0 - W + 1 : jb.ss;
+    b_first = (k_first - jb.ss) / kBKV;
+    nblk = (q_last - jb.ss) / kBKV - b_first + 1;
+}
+
 __global__ void __launch_bounds__(kThreads, 2)
-    attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p) {
+    attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p,
+                             int64_t njobs) {
     using L = AttnLayout;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -153,87 +228,41 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint8_t* smem = smem_raw + (sbase - raw);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // ---- which (sequence, query block) this CTA takes: blocks of sequence s
-    // are numbered from its last (the heaviest under the causal mask) down
-    __shared__ int job[4];  // seq start, seq end, first query, valid
-    if (warp == 0) {
-        const int x = blockIdx.x;
-        int base = 0, found = 0, ss = 0, se = 0, q0 = 0, bad = 0;
-        for (int s0 = 0; s0 < p.nseq && !found; s0 += 32) {
-            const int s = s0 + lane;
-            int a = 0, b = 0, nqb = 0;
-            if (s < p.nseq) {
-                a = p.seq_start[s];
-                b = p.seq_start[s + 1];
-                if (a < 0 || b < a || b > p.M) bad = 1;
-                nqb = b > a ? (b - a + kBQ - 1) / kBQ : 0;
-            }
-            if (__any_sync(0xffffffffu, bad)) {
-                bad = 1;
-                break;
-            }
-            int incl = nqb;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int t = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += t;
-            }
-            const int excl = incl - nqb;
-            const bool mine = s < p.nseq && x >= base + excl && x < base + incl;
-            const unsigned who = __ballot_sync(0xffffffffu, mine);
-            if (who) {
-                const int src = __ffs(who) - 1;
-                const int e = __shfl_sync(0xffffffffu, excl, src);
-                const int n = __shfl_sync(0xffffffffu, nqb, src);
-                ss = __shfl_sync(0xffffffffu, a, src);
-                se = __shfl_sync(0xffffffffu, b, src);
-                const int local = x - base - e;
-                q0 = ss + (n - 1 - local) * kBQ;
-                found = 1;
-            }
-            base += __shfl_sync(0xffffffffu, incl, 31);
-        }
-        if (lane == 0) {
-            if (bad) atomicExch(p.status, 1 /* W4A16_ERR_INVALID_ARG */);
-            job[0] = ss;
-            job[1] = se;
-            job[2] = q0;
-            job[3] = found && !bad;
-        }
-    }
-    __syncthreads();
-    if (!job[3]) return;  // past the last query block (the grid is an upper bound)
-    const int ss = job[0], se = job[1], q0 = job[2];
-    const int h = blockIdx.y;
-    const int W = p.window;
-    // key blocks of the sequence that any query of the block can see
-    const int q_last = (q0 + kBQ - 1 < se - 1 ? q0 + kBQ - 1 : se - 1);
-    const int k_first = q0 - W + 1 > ss ? q0 - W + 1 : ss;
-    const int b_first = (k_first - ss) / kBKV, b_last = (q_last - ss) / kBKV;
-    const int nblk = b_last - b_first + 1;
-
     const uint32_t bars = sbase + L::BAR_OFF;
-    const uint32_t q_full = bars;
-    const uint32_t k_full = bars + 8u, k_empty = bars + 16u;
-    const uint32_t v_full = bars + 24u, v_empty = bars + 32u;
-    const uint32_t s_full = bars + 40u, p_full = bars + 48u;
-    const uint32_t o_ready = bars + 56u, drain = bars + 64u;
+    const uint32_t q_full = bars, q_empty = bars + 8u;
+    const uint32_t k_full = bars + 16u, k_empty = bars + 24u;
+    const uint32_t v_full = bars + 32u, v_empty = bars + 40u;
+    const uint32_t s_full = bars + 48u, p_full = bars + 56u;
+    const uint32_t o_ready = bars + 64u, drain = bars + 72u;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
+    int* bad_flag = reinterpret_cast<int*>(smem + L::MISC_OFF + 8);
 
-    if (threadIdx.x == 0) {
-        mbar_init(q_full, 1);
-        mbar_init(k_full, 1);
-        mbar_init(k_empty, 1);
-        mbar_init(v_full, 1);
-        mbar_init(v_empty, 1);
-        mbar_init(s_full, 1);
-        mbar_init(p_full, 4);  // one arrival per softmax warp
-        mbar_init(o_ready, 1);
-        mbar_init(drain, 1);
-        *abort_flag = 0;
-        fence_mbar_init();
-        prefetch_tmap(&tmap_qkv);
+    if (warp == 0) {
+        // the sequence boundaries must be non-decreasing within [0, M]
+        int bad = 0;
+        for (int s = lane; s < p.nseq; s += 32) {
+            const int a = p.seq_start[s], b = p.seq_start[s + 1];
+            if (a < 0 || b < a || b > p.M) bad = 1;
+        }
+        bad = __any_sync(0xffffffffu, bad);
+        if (lane == 0) {
+            if (bad) atomicExch(p.status, 1 /* W4A16_ERR_INVALID_ARG */);
+            *bad_flag = bad;
+            mbar_init(q_full, 1);
+            mbar_init(q_empty, 1);
+            mbar_init(k_full, 1);
+            mbar_init(k_empty, 1);
+            mbar_init(v_full, 1);
+            mbar_init(v_empty, 1);
+            mbar_init(s_full, 1);
+            mbar_init(p_full, 4);  // one arrival per softmax warp
+            mbar_init(o_ready, 1);
+            mbar_init(drain, 1);
+            *abort_flag = 0;
+            fence_mbar_init();
+            prefetch_tmap(&tmap_qkv);
+        }
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
@@ -244,36 +273,55 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     const int Hd = p.H * kD;
+    const int W = p.window;
+    const int64_t t_first = blockIdx.x, t_step = gridDim.x;
+    const bool run = *bad_flag == 0;
+    JobCursor cur;
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
-        if (lane == 0) {
-            bool ok = true;
-            mbar_arrive_expect_tx(q_full, L::TILE);
-            tma_load_2d(sbase + L::Q_OFF, &tmap_qkv, q_full, h * kD, q0);
-            tma_load_2d(sbase + L::Q_OFF + L::BOX, &tmap_qkv, q_full, h * kD + 64, q0);
-            // K of a block is free once its S product is done, V once its PV
-            // product is: K of block j + 1 loads while block j's softmax runs
-            int nk = 0, nv = 0;
-            for (int j = 0; ok && j < nblk; ++j) {
-                const int row = ss + (b_first + j) * kBKV;
-                if (!wait_one(k_empty, (j & 1u) ^ 1u, abort_flag, p.status)) {
-                    ok = false;
-                    break;
+        // Q of a job loads once the last S product of the previous job is
+        // done; K of a block once the block before's S product is, V once its
+        // PV product is: Q and K of the next job land during the current
+        // job's last softmax and epilogue.
+        bool ok = run;
+        uint32_t g = 0, jn = 0, nk = 0, nv = 0;
+        for (int64_t t = t_first; ok && t < njobs; t += t_step) {
+            const AttnJob jb = job_at(p, t, lane, cur);
+            if (!jb.valid) break;
+            int b_first, nblk;
+            key_range(jb, W, b_first, nblk);
+            if (lane == 0) {
+                if (!wait_one(q_empty, (jn & 1u) ^ 1u, abort_flag, p.status)) ok = false;
+                if (ok) {
+                    mbar_arrive_expect_tx(q_full, L::TILE);
+                    tma_load_2d(sbase + L::Q_OFF, &tmap_qkv, q_full, jb.h * kD, jb.q0);
+                    tma_load_2d(sbase + L::Q_OFF + L::BOX, &tmap_qkv, q_full, jb.h * kD + 64, jb.q0);
                 }
-                mbar_arrive_expect_tx(k_full, L::TILE);
-                tma_load_2d(sbase + L::K_OFF, &tmap_qkv, k_full, Hd + h * kD, row);
-                tma_load_2d(sbase + L::K_OFF + L::BOX, &tmap_qkv, k_full, Hd + h * kD + 64, row);
-                ++nk;
-                if (!wait_one(v_empty, (j & 1u) ^ 1u, abort_flag, p.status)) {
-                    ok = false;
-                    break;
+                for (int j = 0; ok && j < nblk; ++j, ++g) {
+                    const int row = jb.ss + (b_first + j) * kBKV;
+                    if (!wait_one(k_empty, (g & 1u) ^ 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(k_full, L::TILE);
+                    tma_load_2d(sbase + L::K_OFF, &tmap_qkv, k_full, Hd + jb.h * kD, row);
+                    tma_load_2d(sbase + L::K_OFF + L::BOX, &tmap_qkv, k_full, Hd + jb.h * kD + 64, row);
+                    ++nk;
+                    if (!wait_one(v_empty, (g & 1u) ^ 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(v_full, L::TILE);
+                    tma_load_2d(sbase + L::V_OFF, &tmap_qkv, v_full, 2 * Hd + jb.h * kD, row);
+                    tma_load_2d(sbase + L::V_OFF + L::BOX, &tmap_qkv, v_full, 2 * Hd + jb.h * kD + 64, row);
+                    ++nv;
                 }
-                mbar_arrive_expect_tx(v_full, L::TILE);
-                tma_load_2d(sbase + L::V_OFF, &tmap_qkv, v_full, 2 * Hd + h * kD, row);
-                tma_load_2d(sbase + L::V_OFF + L::BOX, &tmap_qkv, v_full, 2 * Hd + h * kD + 64, row);
-                ++nv;
             }
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            ++jn;
+        }
+        if (lane == 0) {
             // every load issued has landed before exit
             auto settle = [&](uint32_t bar, uint32_t parity) {
                 const uint64_t t0 = global_timer_ns();
@@ -281,57 +329,89 @@ __global__ void __launch_bounds__(kThreads, 2)
                     if (global_timer_ns() - t0 > kWaitLimitNs) break;
                 }
             };
-            settle(q_full, 0);
+            if (jn > 0) settle(q_full, (jn - 1) & 1u);
             if (nk > 0) settle(k_full, (nk - 1) & 1u);
             if (nv > 0) settle(v_full, (nv - 1) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
-            constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
-            bool ok = wait_one(q_full, 0, abort_flag, p.status);
-            // S of block j; P of block j - 1 lives in the same columns, so S
-            // waits for that block's PV product to complete
-            auto issue_s = [&](int j) -> bool {
-                if (!wait_one(k_full, j & 1u, abort_flag, p.status)) return false;
-                if (j >= 1 && !wait_one(o_ready, (j - 1) & 1u, abort_flag, p.status)) return false;
-                tc_fence_after();
-                const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF;
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
+        constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
+        bool ok = run;
+        uint32_t g = 0, jn = 0;
+        // S of global block g; P of block g - 1 lives in the same columns, so
+        // S waits for that block's PV product.  The last S of a job frees Q.
+        auto issue_s = [&](uint32_t gb, bool last) -> bool {
+            if (!wait_one(k_full, gb & 1u, abort_flag, p.status)) return false;
+            if (gb >= 1 && !wait_one(o_ready, (gb - 1) & 1u, abort_flag, p.status)) return false;
+            tc_fence_after();
+            const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF;
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
-                    tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
-                              sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
-                }
-                tc_commit(s_full);
-                tc_commit(k_empty);
-                return true;
-            };
-            if (ok && nblk > 0) ok = issue_s(0);
-            for (int j = 0; ok && j < nblk; ++j) {
-                // O += P V once the softmax warps have written P of block j
-                if (!wait_one(p_full, j & 1u, abort_flag, p.status) ||
-                    !wait_one(v_full, j & 1u, abort_flag, p.status)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t vs = sbase + L::V_OFF;
+            for (int kk = 0; kk < kD / 16; ++kk) {
+                const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
+                tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
+                          sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
+            }
+            tc_commit(s_full);
+            tc_commit(k_empty);
+            if (last) tc_commit(q_empty);
+            return true;
+        };
+        AttnJob jb{};
+        int b_first = 0, nblk = 0;
+        if (ok && t_first < njobs) {
+            jb = job_at(p, t_first, lane, cur);
+            if (jb.valid) key_range(jb, W, b_first, nblk);
+        }
+        if (lane == 0 && ok && jb.valid) {
+            ok = wait_one(q_full, 0, abort_flag, p.status) && issue_s(0, nblk == 1);
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        for (int64_t t = t_first; ok && jb.valid; t += t_step) {
+            // the next job, so that its first S product overlaps this job's epilogue
+            AttnJob nx{};
+            int nb_first = 0, nnblk = 0;
+            if (t + t_step < njobs) {
+                nx = job_at(p, t + t_step, lane, cur);
+                if (nx.valid) key_range(nx, W, nb_first, nnblk);
+            }
+            if (lane == 0) {
+                for (int j = 0; ok && j < nblk; ++j, ++g) {
+                    // O += P V once the softmax warps have written P of block j
+                    // (for a job's first block, after they read out the
+                    // previous job's O)
+                    if (!wait_one(p_full, g & 1u, abort_flag, p.status) ||
+                        !wait_one(v_full, g & 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t vs = sbase + L::V_OFF;
 #pragma unroll
-                for (int kk = 0; kk < kBKV / 16; ++kk) {
-                    // keys 16 kk .. 16 kk + 15: rows of the V tile; P columns 8 kk ..
-                    tc_mma_ts(tmem + L::O_COL, tmem + L::P_COL + kk * 8,
-                              sdesc_mnmajor_sw128(vs + kk * 16 * 128, L::BOX, 1024), idesc_o,
-                              (j > 0 || kk > 0) ? 1u : 0u);
-                }
-                tc_commit(o_ready);
-                tc_commit(v_empty);
-                if (j + 1 < nblk && !issue_s(j + 1)) {
-                    ok = false;
-                    break;
+                    for (int kk = 0; kk < kBKV / 16; ++kk) {
+                        // keys 16 kk .. 16 kk + 15: rows of the V tile; P columns 8 kk ..
+                        tc_mma_ts(tmem + L::O_COL, tmem + L::P_COL + kk * 8,
+                                  sdesc_mnmajor_sw128(vs + kk * 16 * 128, L::BOX, 1024), idesc_o,
+                                  (j > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc_commit(o_ready);
+                    tc_commit(v_empty);
+                    if (j + 1 < nblk) {
+                        ok = issue_s(g + 1, j + 2 == nblk);
+                    } else if (nx.valid) {
+                        ok = wait_one(q_full, (jn + 1) & 1u, abort_flag, p.status) &&
+                             issue_s(g + 1, nnblk == 1);
+                    }
                 }
             }
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            g = __shfl_sync(0xffffffffu, g, 0);
+            ++jn;
+            jb = nx;
+            b_first = nb_first;
+            nblk = nnblk;
+        }
+        if (lane == 0) {
             tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
             const uint64_t t0 = global_timer_ns();
             while (!mbar_try_wait(drain, 0)) {
@@ -342,136 +422,164 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ------------------------------------------------------------ softmax + epilogue
         const int sub = warp & 3;  // TMEM sub-partition: lanes 32 sub ..
         const int r = sub * 32 + lane;          // query row within the block
-        const int i = q0 + r;                   // query token
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const float c = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
-        // Running max m (log2 units, scale folded in) and sum l.  The max is
-        // raised lazily: only when a block's max exceeds it by more than 8
-        // (p <= 2^8 otherwise), so O is rescaled rarely; O and l always use
-        // the same m, so the final O / l is exact either way.
-        float m = kMaskedScore, l = 0.0f;
-        bool ok = true;
-        for (int j = 0; ok && j < nblk; ++j) {
-            if (!wait_warp(s_full, j & 1u, abort_flag, p.status)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            const int kbase = ss + (b_first + j) * kBKV;
-            // every key of the block allowed for every query of the block
-            const bool interior = kbase + kBKV - 1 <= q0 && kbase > q0 + kBQ - 1 - W;
-            const uint32_t s_tm = lane_base + L::S_COL;
-            // the row's 128 raw scores, read once; masked keys become -inf, so
-            // their p = 2^(-inf) is exactly 0 with no compare in the exp loop
-            uint32_t v[kBKV / 32][32];
-#pragma unroll
-            for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_32x32b_x32(s_tm + ch * 32, v[ch]);
-#pragma unroll
-            for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_wait(v[ch]);
-            // allowed key offsets in the block for query i: lo .. hi (keys past
-            // the end of the sequence only meet rows past it, never stored)
-            const int hi = i - kbase, lo = i - W + 1 - kbase;
-            // live[ch]: some lane of the warp has an allowed key in chunk ch
-            bool live[kBKV / 32];
-#pragma unroll
-            for (int ch = 0; ch < kBKV / 32; ++ch) {
-                live[ch] = interior || __any_sync(0xffffffffu, hi >= ch * 32 && lo <= ch * 32 + 31);
-                if (!interior && live[ch] &&
-                    __any_sync(0xffffffffu, hi < ch * 32 + 31 || lo > ch * 32)) {
-#pragma unroll
-                    for (int t = 0; t < 32; ++t) {
-                        const int k = ch * 32 + t;
-                        if (k > hi || k < lo) v[ch][t] = 0xFF800000u;
-                    }
-                }
-            }
-            float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-            for (int ch = 0; ch < kBKV / 32; ++ch) {
-                if (!live[ch]) continue;
-#pragma unroll
-                for (int t = 0; t < 32; t += 4) {
-                    mx0 = fmax3(mx0, __uint_as_float(v[ch][t]), __uint_as_float(v[ch][t + 1]));
-                    mx1 = fmax3(mx1, __uint_as_float(v[ch][t + 2]), __uint_as_float(v[ch][t + 3]));
-                }
-            }
-            const float mb = fmaxf(mx0, mx1) * c;  // c > 0
-            const bool raise = mb > m + 8.0f;
-            const float m_new = raise ? mb : m;
-            const float alpha = ex2(m - m_new);
-            const float nm = -m_new;
-            float2 sum = make_float2(0.0f, 0.0f);
-#pragma unroll
-            for (int ch = 0; ch < kBKV / 32; ++ch) {
-                uint32_t pk[16];
-                if (live[ch]) {
-#pragma unroll
-                    for (int t = 0; t < 16; ++t) {
-                        // p = 2^(s c - m) for a key pair: one paired FMA, two ex2
-                        float2 e = ffma2(make_float2(__uint_as_float(v[ch][2 * t]),
-                                                     __uint_as_float(v[ch][2 * t + 1])), c, nm);
-                        e.x = ex2(e.x);
-                        e.y = ex2(e.y);
-                        sum = fadd2(sum, e);
-                        pk[t] = pack_bf16x2_rn(e.x, e.y);
-                    }
-                } else {
-#pragma unroll
-                    for (int t = 0; t < 16; ++t) pk[t] = 0u;
-                }
-                tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
-            }
-            // rescale O (the sum over blocks before j) to the new max; the PV
-            // product of block j-1 has completed, as S of block j followed it
-            if (j > 0) {
-                if (!wait_warp(o_ready, (j - 1) & 1u, abort_flag, p.status)) {
+        bool ok = run;
+        uint32_t g = 0;
+        for (int64_t t = t_first; ok && t < njobs; t += t_step) {
+            const AttnJob jb = job_at(p, t, lane, cur);
+            if (!jb.valid) break;
+            int b_first, nblk;
+            key_range(jb, W, b_first, nblk);
+            const int i = jb.q0 + r;  // query token
+            // Running max m (log2 units, scale folded in) and sum l.  The max is
+            // raised lazily: only when a block's max exceeds it by more than 8
+            // (p <= 2^8 otherwise), so O is rescaled rarely; O and l always use
+            // the same m, so the final O / l is exact either way.
+            float m = kMaskedScore, l = 0.0f;
+            for (int j = 0; ok && j < nblk; ++j, ++g) {
+                if (!wait_warp(s_full, g & 1u, abort_flag, p.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, raise)) {
-#pragma unroll 1
-                    for (int ch = 0; ch < kD / 32; ++ch) {
-                        uint32_t o[32];
-                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
-                        tmem_ld_wait(o);
+                const int kbase = jb.ss + (b_first + j) * kBKV;
+                // every key of the block allowed for every query of the block
+                const bool interior = kbase + kBKV - 1 <= jb.q0 && kbase > jb.q0 + kBQ - 1 - W;
+                const uint32_t s_tm = lane_base + L::S_COL;
+                // the row's 128 raw scores, read once; masked keys become -inf, so
+                // their p = 2^(-inf) is exactly 0 with no compare in the exp loop
+                uint32_t v[kBKV / 32][32];
 #pragma unroll
-                        for (int t = 0; t < 32; ++t)
-                            o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
-                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_32x32b_x32(s_tm + ch * 32, v[ch]);
+#pragma unroll
+                for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_wait(v[ch]);
+                // allowed key offsets in the block for query i: lo .. hi (keys past
+                // the end of the sequence only meet rows past it, never stored)
+                const int hi = i - kbase, lo = i - W + 1 - kbase;
+                // live[ch]: some lane of the warp has an allowed key in chunk ch
+                bool live[kBKV / 32];
+#pragma unroll
+                for (int ch = 0; ch < kBKV / 32; ++ch) {
+                    live[ch] = interior || __any_sync(0xffffffffu, hi >= ch * 32 && lo <= ch * 32 + 31);
+                    if (!interior && live[ch] &&
+                        __any_sync(0xffffffffu, hi < ch * 32 + 31 || lo > ch * 32)) {
+#pragma unroll
+                        for (int t = 0; t < 32; ++t) {
+                            const int k = ch * 32 + t;
+                            if (k > hi || k < lo) v[ch][t] = 0xFF800000u;
+                        }
                     }
                 }
+                float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                for (int ch = 0; ch < kBKV / 32; ++ch) {
+                    if (!live[ch]) continue;
+#pragma unroll
+                    for (int t = 0; t < 32; t += 8) {
+#pragma unroll
+                        for (int u = 0; u < 4; ++u)
+                            mx[u] = fmax3(mx[u], __uint_as_float(v[ch][t + 2 * u]),
+                                          __uint_as_float(v[ch][t + 2 * u + 1]));
+                    }
+                }
+                const float mb = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c;  // c > 0
+                const bool raise = mb > m + 8.0f;
+                const float m_new = raise ? mb : m;
+                const float alpha = ex2(m - m_new);
+                const float nm = -m_new;
+                float2 sum[2] = {make_float2(0.0f, 0.0f), make_float2(0.0f, 0.0f)};
+#pragma unroll
+                for (int ch = 0; ch < kBKV / 32; ++ch) {
+                    uint32_t pk[16];
+                    if (live[ch]) {
+#pragma unroll
+                        for (int t = 0; t < 16; ++t) {
+                            // p = 2^(s c - m) for a key pair: one paired FMA, two ex2
+                            float2 e = ffma2(make_float2(__uint_as_float(v[ch][2 * t]),
+                                                         __uint_as_float(v[ch][2 * t + 1])), c, nm);
+                            e.x = ex2(e.x);
+                            e.y = ex2(e.y);
+                            sum[t & 1] = fadd2(sum[t & 1], e);
+                            pk[t] = pack_bf16x2_rn(e.x, e.y);
+                        }
+                    } else {
+#pragma unroll
+                        for (int t = 0; t < 16; ++t) pk[t] = 0u;
+                    }
+                    tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
+                }
+                // rescale O (the sum over blocks before j) to the new max; the PV
+                // product of block j-1 has completed, as S of block j followed it
+                if (j > 0) {
+                    if (!wait_warp(o_ready, (g - 1) & 1u, abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    if (__any_sync(0xffffffffu, raise)) {
+#pragma unroll 1
+                        for (int ch = 0; ch < kD / 32; ++ch) {
+                            uint32_t o[32];
+                            tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                            tmem_ld_wait(o);
+#pragma unroll
+                            for (int t = 0; t < 32; ++t)
+                                o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
+                            tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                        }
+                    }
+                }
+                l = l * alpha + ((sum[0].x + sum[1].x) + (sum[0].y + sum[1].y));
+                m = m_new;
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(p_full);  // P of block j written over S
             }
-            l = l * alpha + (sum.x + sum.y);
-            m = m_new;
-            tmem_st_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(p_full);  // P of block j written over S
-        }
-        // ---- epilogue: O / l -> bf16
-        if (ok && nblk > 0 && wait_warp(o_ready, (nblk - 1) & 1u, abort_flag, p.status)) {
+            // ---- epilogue: O / l -> bf16.  The next job's first PV product,
+            // which overwrites O, waits for P of that job, which these warps
+            // write only after this epilogue has read O.
+            if (!ok || !wait_warp(o_ready, (g - 1) & 1u, abort_flag, p.status)) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
             const float inv = l > 0.0f ? 1.0f / l : 0.0f;
-            __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out) +
-                                  static_cast<int64_t>(i) * Hd + h * kD;
+            // Each 32-column chunk goes through the warp's staging buffer, so
+            // that a store instruction writes 8 rows x 64 contiguous bytes
+            // rather than 32 rows x 16: 16-byte unit u of row q sits at unit
+            // u ^ ((q >> 1) & 3), which keeps both sides at the minimum of
+            // four shared-memory wavefronts.
+            uint8_t* stage = smem + L::STAGE_OFF + sub * L::STAGE_WARP;
+            const int rows_left = jb.se - (jb.q0 + sub * 32);  // rows of this warp to store
+            __nv_bfloat16* obase = reinterpret_cast<__nv_bfloat16*>(p.out) +
+                                   static_cast<int64_t>(jb.q0 + sub * 32) * Hd + jb.h * kD;
 #pragma unroll 1
             for (int ch = 0; ch < kD / 32; ++ch) {
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, v);
-                tmem_ld_wait(v);
-                if (i < se) {
-                    uint4* dst = reinterpret_cast<uint4*>(orow + ch * 32);
+                uint32_t o[32];
+                tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                tmem_ld_wait(o);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 w;
-                        w.x = pack_bf16x2_rn(__uint_as_float(v[8 * q + 0]) * inv, __uint_as_float(v[8 * q + 1]) * inv);
-                        w.y = pack_bf16x2_rn(__uint_as_float(v[8 * q + 2]) * inv, __uint_as_float(v[8 * q + 3]) * inv);
-                        w.z = pack_bf16x2_rn(__uint_as_float(v[8 * q + 4]) * inv, __uint_as_float(v[8 * q + 5]) * inv);
-                        w.w = pack_bf16x2_rn(__uint_as_float(v[8 * q + 6]) * inv, __uint_as_float(v[8 * q + 7]) * inv);
-                        dst[q] = w;
-                    }
+                for (int u = 0; u < 4; ++u) {
+                    const uint32_t* w8 = &o[8 * u];
+                    uint4 w;
+                    w.x = pack_bf16x2_rn(__uint_as_float(w8[0]) * inv, __uint_as_float(w8[1]) * inv);
+                    w.y = pack_bf16x2_rn(__uint_as_float(w8[2]) * inv, __uint_as_float(w8[3]) * inv);
+                    w.z = pack_bf16x2_rn(__uint_as_float(w8[4]) * inv, __uint_as_float(w8[5]) * inv);
+                    w.w = pack_bf16x2_rn(__uint_as_float(w8[6]) * inv, __uint_as_float(w8[7]) * inv);
+                    *reinterpret_cast<uint4*>(stage + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) = w;
                 }
+                __syncwarp();
+#pragma unroll
+                for (int it = 0; it < 4; ++it) {
+                    const int q = it * 8 + (lane >> 2), u = lane & 3;
+                    const uint4 w = *reinterpret_cast<const uint4*>(stage + q * 64 +
+                                                                    ((u ^ ((q >> 1) & 3)) << 4));
+                    if (q < rows_left)
+                        *reinterpret_cast<uint4*>(obase + static_cast<int64_t>(q) * Hd + ch * 32 + u * 8) = w;
+                }
+                __syncwarp();
             }
         }
     }
@@ -492,8 +600,16 @@ cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnPara
     if (e != cudaSuccess) return e;
     // upper bound on the query blocks: sum over sequences of ceil(len / 128)
     const int64_t qblocks = (static_cast<int64_t>(p.M) + kBQ - 1) / kBQ + p.nseq;
-    const dim3 grid(static_cast<unsigned>(qblocks), static_cast<unsigned>(p.H));
-    attention_prefill_kernel<<<grid, kThreads, L::SMEM_BYTES, stream>>>(*tmap_qkv, p);
+    const int64_t njobs = qblocks * p.H;
+    // persistent: two CTAs per SM, each taking every grid-th job
+    int dev = 0, sms = 0;
+    e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int64_t grid = njobs < 2 * static_cast<int64_t>(sms) ? njobs : 2 * static_cast<int64_t>(sms);
+    attention_prefill_kernel<<<static_cast<unsigned>(grid), kThreads, L::SMEM_BYTES, stream>>>(
+        *tmap_qkv, p, njobs);
     return cudaGetLastError();
 }
 
