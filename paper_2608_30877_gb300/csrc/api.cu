@@ -425,8 +425,12 @@ extern "C" int w4a16_attention_prefill(const void* qkv_bf16, const void* seq_sta
     int rc = device_state(&st);
     if (rc != W4A16_OK) return rc;
     alignas(64) CUtensorMap tq;
+    alignas(64) CUtensorMap tkv;
     rc = encode_2d(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, qkv_bf16, 3 * H * d, M, 3 * H * d * 2,
                    64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != W4A16_OK) return rc;
+    rc = encode_2d(&tkv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, qkv_bf16, 3 * H * d, M, 3 * H * d * 2,
+                   64, attention_key_block(), CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != W4A16_OK) return rc;
     AttnParams p;
     p.seq_start = static_cast<const int32_t*>(seq_start_i32);
@@ -437,7 +441,7 @@ extern "C" int w4a16_attention_prefill(const void* qkv_bf16, const void* seq_sta
     p.nseq = static_cast<int>(nseq);
     p.window = window > kMaxDim ? static_cast<int>(kMaxDim) : static_cast<int>(window);
     p.scale = 1.0f / sqrtf(static_cast<float>(d));
-    return launch_attention_prefill(&tq, p, static_cast<cudaStream_t>(stream)) == cudaSuccess
+    return launch_attention_prefill(&tq, &tkv, p, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? W4A16_OK
                : W4A16_ERR_CUDA;
 }

@@ -38,28 +38,31 @@ namespace w4a16 {
 namespace {
 
 constexpr int kD = 128;        // head dimension
-constexpr int kBQ = 128;       // queries per CTA (MMA M)
-constexpr int kBKV = 128;      // keys per block (MMA N of S, K of PV)
+constexpr int kBQ = 128;       // queries per job (MMA M)
+constexpr int kBKV = 64;       // keys per block (MMA N of S, K of PV)
 constexpr int kThreads = 6 * 32;  // TMA warp, MMA warp, 4 softmax warps
 
 struct AttnLayout {
-    static constexpr int BOX = kBQ * 64 * 2;       // one [128 rows x 64 cols] bf16 box: 16 KB
-    static constexpr int TILE = 2 * BOX;           // [128 x 128]: 32 KB
+    static constexpr int QBOX = kBQ * 128;    // one [128 rows x 64 cols] bf16 box: 16 KB
+    static constexpr int KBOX = kBKV * 128;   // one [64 rows x 64 cols] bf16 box: 8 KB
+    static constexpr int Q_TILE = 2 * QBOX;   // [128 x 128]: 32 KB
+    static constexpr int KV_TILE = 2 * KBOX;  // [64 x 128]: 16 KB
     static constexpr int Q_OFF = 0;
-    static constexpr int K_OFF = Q_OFF + TILE;
-    static constexpr int V_OFF = K_OFF + TILE;
+    static constexpr int K_OFF = Q_OFF + Q_TILE;       // two stages
+    static constexpr int V_OFF = K_OFF + 2 * KV_TILE;  // two stages
     // epilogue staging: per softmax warp 32 rows x 32 columns of bf16 output
-    static constexpr int STAGE_OFF = V_OFF + TILE;
+    static constexpr int STAGE_OFF = V_OFF + 2 * KV_TILE;
     static constexpr int STAGE_WARP = 32 * 64;
     static constexpr int BAR_OFF = STAGE_OFF + 4 * STAGE_WARP;
-    // q_full, q_empty, k_full, k_empty, v_full, v_empty, s_full, p_full,
-    // o_ready, drain
-    static constexpr int NBARS = 10;
+    // q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2],
+    // s_full[2], p_full[2], o_ready[2], drain
+    static constexpr int NBARS = 17;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
-    // tensor memory columns: S, with P written over it in place, and O; 256
-    // columns and under 113 KB of shared memory let two CTAs share an SM
-    static constexpr int S_COL = 0, P_COL = 0, O_COL = 128, TMEM_COLS = 256;
+    // tensor memory columns: two S buffers (blocks alternate; P of a block is
+    // written over the first half of its S) and O
+    static constexpr int S_COL = 0, O_COL = 2 * kBKV, TMEM_COLS = 256;
+    static_assert(O_COL + kD <= TMEM_COLS, "tensor memory");
     // two CTAs per SM: 228 KB per SM, 1 KB of it reserved per CTA
     static_assert(2 * (SMEM_BYTES + 1024) <= 228 * 1024, "shared memory");
 };
@@ -218,8 +221,40 @@ __device__ __forceinline__ void key_range(const AttnJob& jb, int W, int& b_first
     nblk = (q_last - jb.ss) / kBKV - b_first + 1;
 }
 
+// Walks the CTA's key blocks in order across its jobs; warp-collective (the
+// job search uses the whole warp).
+struct BlockWalk {
+    JobCursor cur;
+    int64_t t = 0;
+    AttnJob jb{};
+    int b_first = 0, nblk = 0, j = 0;
+    uint32_t jn = 0;  // jobs of the CTA before this one
+    bool valid = false;
+};
+
+__device__ __forceinline__ void walk_job(const AttnParams& p, int64_t njobs, int lane, BlockWalk& w) {
+    w.valid = false;
+    if (w.t < njobs) {
+        w.jb = job_at(p, w.t, lane, w.cur);
+        if (w.jb.valid) {
+            key_range(w.jb, p.window, w.b_first, w.nblk);
+            w.j = 0;
+            w.valid = true;
+        }
+    }
+}
+
+__device__ __forceinline__ void walk_next(const AttnParams& p, int64_t njobs, int64_t step,
+                                          int lane, BlockWalk& w) {
+    if (++w.j < w.nblk) return;
+    w.t += step;
+    ++w.jn;
+    walk_job(p, njobs, lane, w);
+}
+
 __global__ void __launch_bounds__(kThreads, 2)
-    attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_qkv, const AttnParams p,
+    attention_prefill_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                             const __grid_constant__ CUtensorMap tmap_kv, const AttnParams p,
                              int64_t njobs) {
     using L = AttnLayout;
     extern __shared__ uint8_t smem_raw[];
@@ -230,10 +265,20 @@ __global__ void __launch_bounds__(kThreads, 2)
 
     const uint32_t bars = sbase + L::BAR_OFF;
     const uint32_t q_full = bars, q_empty = bars + 8u;
-    const uint32_t k_full = bars + 16u, k_empty = bars + 24u;
-    const uint32_t v_full = bars + 32u, v_empty = bars + 40u;
-    const uint32_t s_full = bars + 48u, p_full = bars + 56u;
-    const uint32_t o_ready = bars + 64u, drain = bars + 72u;
+    auto k_full = [&](uint32_t s) { return bars + 16u + 8u * s; };
+    auto k_empty = [&](uint32_t s) { return bars + 32u + 8u * s; };
+    auto v_full = [&](uint32_t s) { return bars + 48u + 8u * s; };
+    auto v_empty = [&](uint32_t s) { return bars + 64u + 8u * s; };
+    auto s_full = [&](uint32_t b) { return bars + 80u + 8u * b; };
+    // The barriers of block g are those of index g & 1 and complete once per
+    // two blocks.  A parity wait is unambiguous only while its barrier is at
+    // most one completion ahead or behind the awaited one; with S two blocks
+    // ahead of PV, the softmax may finish P of block g + 1 before the MMA
+    // warp takes P of block g (hence two p_full), and the softmax waits for
+    // PV products only now and then (hence two o_ready).
+    auto p_full = [&](uint32_t b) { return bars + 96u + 8u * b; };
+    auto o_ready = [&](uint32_t b) { return bars + 112u + 8u * b; };
+    const uint32_t drain = bars + 128u;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
     int* bad_flag = reinterpret_cast<int*>(smem + L::MISC_OFF + 8);
@@ -251,17 +296,20 @@ __global__ void __launch_bounds__(kThreads, 2)
             *bad_flag = bad;
             mbar_init(q_full, 1);
             mbar_init(q_empty, 1);
-            mbar_init(k_full, 1);
-            mbar_init(k_empty, 1);
-            mbar_init(v_full, 1);
-            mbar_init(v_empty, 1);
-            mbar_init(s_full, 1);
-            mbar_init(p_full, 4);  // one arrival per softmax warp
-            mbar_init(o_ready, 1);
+            for (uint32_t i = 0; i < 2; ++i) {
+                mbar_init(k_full(i), 1);
+                mbar_init(k_empty(i), 1);
+                mbar_init(v_full(i), 1);
+                mbar_init(v_empty(i), 1);
+                mbar_init(s_full(i), 1);
+                mbar_init(p_full(i), 4);  // one arrival per softmax warp
+                mbar_init(o_ready(i), 1);
+            }
             mbar_init(drain, 1);
             *abort_flag = 0;
             fence_mbar_init();
-            prefetch_tmap(&tmap_qkv);
+            prefetch_tmap(&tmap_q);
+            prefetch_tmap(&tmap_kv);
         }
     }
     if (warp == 1) {
@@ -276,15 +324,16 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int W = p.window;
     const int64_t t_first = blockIdx.x, t_step = gridDim.x;
     const bool run = *bad_flag == 0;
-    JobCursor cur;
 
+    // Global block g of the CTA (counted across its jobs) uses K/V stage and
+    // S buffer g & 1; each of those barriers completes once per two blocks.
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         // Q of a job loads once the last S product of the previous job is
-        // done; K of a block once the block before's S product is, V once its
-        // PV product is: Q and K of the next job land during the current
-        // job's last softmax and epilogue.
+        // done; K of block g once the S product of block g - 2 is, V once its
+        // PV product is.
         bool ok = run;
+        JobCursor cur;
         uint32_t g = 0, jn = 0, nk = 0, nv = 0;
         for (int64_t t = t_first; ok && t < njobs; t += t_step) {
             const AttnJob jb = job_at(p, t, lane, cur);
@@ -294,27 +343,30 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) {
                 if (!wait_one(q_empty, (jn & 1u) ^ 1u, abort_flag, p.status)) ok = false;
                 if (ok) {
-                    mbar_arrive_expect_tx(q_full, L::TILE);
-                    tma_load_2d(sbase + L::Q_OFF, &tmap_qkv, q_full, jb.h * kD, jb.q0);
-                    tma_load_2d(sbase + L::Q_OFF + L::BOX, &tmap_qkv, q_full, jb.h * kD + 64, jb.q0);
+                    mbar_arrive_expect_tx(q_full, L::Q_TILE);
+                    tma_load_2d(sbase + L::Q_OFF, &tmap_q, q_full, jb.h * kD, jb.q0);
+                    tma_load_2d(sbase + L::Q_OFF + L::QBOX, &tmap_q, q_full, jb.h * kD + 64, jb.q0);
                 }
                 for (int j = 0; ok && j < nblk; ++j, ++g) {
+                    const uint32_t s = g & 1u, par = ((g >> 1) & 1u) ^ 1u;
                     const int row = jb.ss + (b_first + j) * kBKV;
-                    if (!wait_one(k_empty, (g & 1u) ^ 1u, abort_flag, p.status)) {
+                    const uint32_t ks = sbase + L::K_OFF + s * L::KV_TILE;
+                    const uint32_t vs = sbase + L::V_OFF + s * L::KV_TILE;
+                    if (!wait_one(k_empty(s), par, abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(k_full, L::TILE);
-                    tma_load_2d(sbase + L::K_OFF, &tmap_qkv, k_full, Hd + jb.h * kD, row);
-                    tma_load_2d(sbase + L::K_OFF + L::BOX, &tmap_qkv, k_full, Hd + jb.h * kD + 64, row);
+                    mbar_arrive_expect_tx(k_full(s), L::KV_TILE);
+                    tma_load_2d(ks, &tmap_kv, k_full(s), Hd + jb.h * kD, row);
+                    tma_load_2d(ks + L::KBOX, &tmap_kv, k_full(s), Hd + jb.h * kD + 64, row);
                     ++nk;
-                    if (!wait_one(v_empty, (g & 1u) ^ 1u, abort_flag, p.status)) {
+                    if (!wait_one(v_empty(s), par, abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(v_full, L::TILE);
-                    tma_load_2d(sbase + L::V_OFF, &tmap_qkv, v_full, 2 * Hd + jb.h * kD, row);
-                    tma_load_2d(sbase + L::V_OFF + L::BOX, &tmap_qkv, v_full, 2 * Hd + jb.h * kD + 64, row);
+                    mbar_arrive_expect_tx(v_full(s), L::KV_TILE);
+                    tma_load_2d(vs, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD, row);
+                    tma_load_2d(vs + L::KBOX, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD + 64, row);
                     ++nv;
                 }
             }
@@ -330,86 +382,77 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             };
             if (jn > 0) settle(q_full, (jn - 1) & 1u);
-            if (nk > 0) settle(k_full, (nk - 1) & 1u);
-            if (nv > 0) settle(v_full, (nv - 1) & 1u);
+            for (uint32_t i = nk > 2 ? nk - 2 : 0; i < nk; ++i) settle(k_full(i & 1u), (i >> 1) & 1u);
+            for (uint32_t i = nv > 2 ? nv - 2 : 0; i < nv; ++i) settle(v_full(i & 1u), (i >> 1) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
+        // S runs two blocks ahead of PV: S of block g + 2 goes into S buffer
+        // g & 1 as soon as the PV product of block g has read P from it, so it
+        // overlaps the softmax of block g + 1.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
         constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
         bool ok = run;
-        uint32_t g = 0, jn = 0;
-        // S of global block g; P of block g - 1 lives in the same columns, so
-        // S waits for that block's PV product.  The last S of a job frees Q.
-        auto issue_s = [&](uint32_t gb, bool last) -> bool {
-            if (!wait_one(k_full, gb & 1u, abort_flag, p.status)) return false;
-            if (gb >= 1 && !wait_one(o_ready, (gb - 1) & 1u, abort_flag, p.status)) return false;
+        auto issue_s = [&](const BlockWalk& w, uint32_t gs) -> bool {
+            const uint32_t b = gs & 1u;
+            if (w.j == 0 && !wait_one(q_full, w.jn & 1u, abort_flag, p.status)) return false;
+            if (!wait_one(k_full(b), (gs >> 1) & 1u, abort_flag, p.status)) return false;
             tc_fence_after();
-            const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF;
+            const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + b * L::KV_TILE;
 #pragma unroll
             for (int kk = 0; kk < kD / 16; ++kk) {
-                const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
-                tc_mma_ss(tmem + L::S_COL, sdesc_kmajor_sw128(qs + off),
-                          sdesc_kmajor_sw128(ks + off), idesc_s, kk > 0 ? 1u : 0u);
+                tc_mma_ss(tmem + L::S_COL + b * kBKV,
+                          sdesc_kmajor_sw128(qs + (kk >> 2) * L::QBOX + (kk & 3) * 32),
+                          sdesc_kmajor_sw128(ks + (kk >> 2) * L::KBOX + (kk & 3) * 32), idesc_s,
+                          kk > 0 ? 1u : 0u);
             }
-            tc_commit(s_full);
-            tc_commit(k_empty);
-            if (last) tc_commit(q_empty);
+            tc_commit(s_full(b));
+            tc_commit(k_empty(b));
+            if (w.j == w.nblk - 1) tc_commit(q_empty);  // the job's last S product frees Q
             return true;
         };
-        AttnJob jb{};
-        int b_first = 0, nblk = 0;
-        if (ok && t_first < njobs) {
-            jb = job_at(p, t_first, lane, cur);
-            if (jb.valid) key_range(jb, W, b_first, nblk);
+        BlockWalk ws, wp;  // the next block to take its S product, the next for its PV product
+        if (ok) {
+            ws.t = t_first;
+            walk_job(p, njobs, lane, ws);
+            wp = ws;
         }
-        if (lane == 0 && ok && jb.valid) {
-            ok = wait_one(q_full, 0, abort_flag, p.status) && issue_s(0, nblk == 1);
+        uint32_t gs = 0, g = 0;
+        for (int k = 0; k < 2 && ok && ws.valid; ++k, ++gs) {
+            if (lane == 0) ok = issue_s(ws, gs);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            walk_next(p, njobs, t_step, lane, ws);
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        for (int64_t t = t_first; ok && jb.valid; t += t_step) {
-            // the next job, so that its first S product overlaps this job's epilogue
-            AttnJob nx{};
-            int nb_first = 0, nnblk = 0;
-            if (t + t_step < njobs) {
-                nx = job_at(p, t + t_step, lane, cur);
-                if (nx.valid) key_range(nx, W, nb_first, nnblk);
-            }
+        while (ok && wp.valid) {
+            const uint32_t b = g & 1u;
             if (lane == 0) {
-                for (int j = 0; ok && j < nblk; ++j, ++g) {
-                    // O += P V once the softmax warps have written P of block j
-                    // (for a job's first block, after they read out the
-                    // previous job's O)
-                    if (!wait_one(p_full, g & 1u, abort_flag, p.status) ||
-                        !wait_one(v_full, g & 1u, abort_flag, p.status)) {
-                        ok = false;
-                        break;
-                    }
+                // O += P V once the softmax warps have written P of block g (for
+                // a job's first block, after they read out the previous job's O)
+                ok = wait_one(p_full(b), (g >> 1) & 1u, abort_flag, p.status) &&
+                     wait_one(v_full(b), (g >> 1) & 1u, abort_flag, p.status);
+                if (ok) {
                     tc_fence_after();
-                    const uint32_t vs = sbase + L::V_OFF;
+                    const uint32_t vs = sbase + L::V_OFF + b * L::KV_TILE;
 #pragma unroll
                     for (int kk = 0; kk < kBKV / 16; ++kk) {
                         // keys 16 kk .. 16 kk + 15: rows of the V tile; P columns 8 kk ..
-                        tc_mma_ts(tmem + L::O_COL, tmem + L::P_COL + kk * 8,
-                                  sdesc_mnmajor_sw128(vs + kk * 16 * 128, L::BOX, 1024), idesc_o,
-                                  (j > 0 || kk > 0) ? 1u : 0u);
+                        tc_mma_ts(tmem + L::O_COL, tmem + L::S_COL + b * kBKV + kk * 8,
+                                  sdesc_mnmajor_sw128(vs + kk * 16 * 128, L::KBOX, 1024), idesc_o,
+                                  (wp.j > 0 || kk > 0) ? 1u : 0u);
                     }
-                    tc_commit(o_ready);
-                    tc_commit(v_empty);
-                    if (j + 1 < nblk) {
-                        ok = issue_s(g + 1, j + 2 == nblk);
-                    } else if (nx.valid) {
-                        ok = wait_one(q_full, (jn + 1) & 1u, abort_flag, p.status) &&
-                             issue_s(g + 1, nnblk == 1);
-                    }
+                    tc_commit(o_ready(b));
+                    tc_commit(v_empty(b));
                 }
+                if (ok && ws.valid)
+                    ok = wait_one(o_ready(b), (g >> 1) & 1u, abort_flag, p.status) && issue_s(ws, gs);
             }
             ok = __shfl_sync(0xffffffffu, ok, 0);
-            g = __shfl_sync(0xffffffffu, g, 0);
-            ++jn;
-            jb = nx;
-            b_first = nb_first;
-            nblk = nnblk;
+            if (ws.valid) {
+                ++gs;
+                walk_next(p, njobs, t_step, lane, ws);
+            }
+            ++g;
+            walk_next(p, njobs, t_step, lane, wp);
         }
         if (lane == 0) {
             tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
@@ -425,6 +468,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const float c = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
         bool ok = run;
+        JobCursor cur;
         uint32_t g = 0;
         for (int64_t t = t_first; ok && t < njobs; t += t_step) {
             const AttnJob jb = job_at(p, t, lane, cur);
@@ -438,7 +482,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             // the same m, so the final O / l is exact either way.
             float m = kMaskedScore, l = 0.0f;
             for (int j = 0; ok && j < nblk; ++j, ++g) {
-                if (!wait_warp(s_full, g & 1u, abort_flag, p.status)) {
+                const uint32_t b = g & 1u;
+                if (!wait_warp(s_full(b), (g >> 1) & 1u, abort_flag, p.status)) {
                     ok = false;
                     break;
                 }
@@ -446,8 +491,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const int kbase = jb.ss + (b_first + j) * kBKV;
                 // every key of the block allowed for every query of the block
                 const bool interior = kbase + kBKV - 1 <= jb.q0 && kbase > jb.q0 + kBQ - 1 - W;
-                const uint32_t s_tm = lane_base + L::S_COL;
-                // the row's 128 raw scores, read once; masked keys become -inf, so
+                const uint32_t s_tm = lane_base + L::S_COL + b * kBKV;
+                // the row's scores, read once; masked keys become -inf, so
                 // their p = 2^(-inf) is exactly 0 with no compare in the exp loop
                 uint32_t v[kBKV / 32][32];
 #pragma unroll
@@ -507,27 +552,25 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
                         for (int t = 0; t < 16; ++t) pk[t] = 0u;
                     }
-                    tmem_st_32x32b_x16(lane_base + L::P_COL + ch * 16, pk);
+                    tmem_st_32x32b_x16(s_tm + ch * 16, pk);
                 }
-                // rescale O (the sum over blocks before j) to the new max; the PV
-                // product of block j-1 has completed, as S of block j followed it
-                if (j > 0) {
-                    if (!wait_warp(o_ready, (g - 1) & 1u, abort_flag, p.status)) {
+                // rescale O (the sum over the job's blocks before j) to the new
+                // max, once the PV product of block g - 1 has completed
+                if (j > 0 && __any_sync(0xffffffffu, raise)) {
+                    if (!wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    if (__any_sync(0xffffffffu, raise)) {
 #pragma unroll 1
-                        for (int ch = 0; ch < kD / 32; ++ch) {
-                            uint32_t o[32];
-                            tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
-                            tmem_ld_wait(o);
+                    for (int ch = 0; ch < kD / 32; ++ch) {
+                        uint32_t o[32];
+                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                        tmem_ld_wait(o);
 #pragma unroll
-                            for (int t = 0; t < 32; ++t)
-                                o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
-                            tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
-                        }
+                        for (int t = 0; t < 32; ++t)
+                            o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
+                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
                     }
                 }
                 l = l * alpha + ((sum[0].x + sum[1].x) + (sum[0].y + sum[1].y));
@@ -535,12 +578,12 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(p_full);  // P of block j written over S
+                if (lane == 0) mbar_arrive(p_full(b));  // P of block g written over its S
             }
             // ---- epilogue: O / l -> bf16.  The next job's first PV product,
             // which overwrites O, waits for P of that job, which these warps
             // write only after this epilogue has read O.
-            if (!ok || !wait_warp(o_ready, (g - 1) & 1u, abort_flag, p.status)) {
+            if (!ok || !wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status)) {
                 ok = false;
                 break;
             }
@@ -591,8 +634,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 
 }  // namespace
 
-cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnParams& p,
-                                     cudaStream_t stream) {
+cudaError_t launch_attention_prefill(const CUtensorMap* tmap_q, const CUtensorMap* tmap_kv,
+                                     const AttnParams& p, cudaStream_t stream) {
     using L = AttnLayout;
     cudaError_t e = cudaFuncSetAttribute(attention_prefill_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -609,10 +652,11 @@ cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnPara
     if (e != cudaSuccess) return e;
     const int64_t grid = njobs < 2 * static_cast<int64_t>(sms) ? njobs : 2 * static_cast<int64_t>(sms);
     attention_prefill_kernel<<<static_cast<unsigned>(grid), kThreads, L::SMEM_BYTES, stream>>>(
-        *tmap_qkv, p, njobs);
+        *tmap_q, *tmap_kv, p, njobs);
     return cudaGetLastError();
 }
 
 int attention_head_dim() { return kD; }
+int attention_key_block() { return kBKV; }
 
 }  // namespace w4a16

@@ -72,8 +72,12 @@ struct AttnParams {
     float scale;               // 1 / sqrt(head dim)
 };
 int attention_head_dim();
-cudaError_t launch_attention_prefill(const CUtensorMap* tmap_qkv, const AttnParams& p,
-                                     cudaStream_t stream);
+// tmap_q: qkv with [128 tokens x 64 features] boxes; tmap_kv: the same
+// tensor with [attention_key_block() tokens x 64 features] boxes (both with
+// the 128-byte swizzle)
+int attention_key_block();
+cudaError_t launch_attention_prefill(const CUtensorMap* tmap_q, const CUtensorMap* tmap_kv,
+                                     const AttnParams& p, cudaStream_t stream);
 
 // Scoring readout (readout.cu).
 constexpr int kTopkMaxK = 1024;  // largest k of the top-k
