@@ -7,9 +7,10 @@
 //   j in the sequence of i, i - W < j <= i;  d = 128.
 //
 // A job is one (128-query block, head), flash-attention style on the
-// 5th-generation tensor core:
+// 5th-generation tensor core, over blocks of 64 keys:
 //   S  = Q K^T   tcgen05.mma kind::f16, A = Q and B = K from shared memory
-//                (TMA, 128-byte swizzle, K-major), S fp32 in tensor memory;
+//                (TMA, 128-byte swizzle, K-major), S fp32 in tensor memory,
+//                two S buffers that blocks alternate between;
 //   softmax      four warps, thread = query row: tcgen05.ld of its S row into
 //                registers, causal/window mask per 32-key chunk, running max
 //                and sum in fp32 (exp2 with the scale folded in), P as bf16
@@ -18,14 +19,16 @@
 //   O += P V     tcgen05.mma with A = P from tensor memory and B = V from
 //                shared memory as an MN-major operand (V is stored token-
 //                major, d contiguous -- exactly the layout the TMA box has);
-//   epilogue     O / l, bf16, 16-byte stores.
-// The kernel is persistent with two CTAs per SM (256 tensor-memory columns
-// and 96 KB of shared memory each), every CTA taking every grid-th job, heads
-// fastest; one CTA's softmax and epilogue overlap the other's MMAs.  Within a
-// CTA the roles are one TMA warp, one MMA warp and the four softmax warps,
-// linked by mbarriers whose phases run on across jobs: Q and K of the next
-// job load during the current job's last softmax, and its first S product
-// runs during the current job's epilogue.
+//   epilogue     O / l, bf16, staged through shared memory for coalesced
+//                stores.
+// S runs two blocks ahead of PV, so the S product of the next block is
+// ready when the softmax of the current one ends.  The kernel is persistent
+// with two CTAs per SM (256 tensor-memory columns and 104 KB of shared memory
+// each), every CTA taking every grid-th job, heads fastest; one CTA's softmax
+// and epilogue overlap the other's MMAs.  Within a CTA the roles are one TMA
+// warp, one MMA warp and the four softmax warps, linked by mbarriers whose
+// phases run on across jobs: Q and K of the next job load during the current
+// job's last blocks, and its first S products run during the epilogue.
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, waits for its own copies and MMAs and frees tensor memory.
 #include "internal.h"
