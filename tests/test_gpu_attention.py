@@ -90,3 +90,31 @@ def test_attention_full_size_sampled_rows():
     gpu = out[torch.from_numpy(rows).cuda()].float().cpu().numpy().astype(np.float64)
     v = O.bf16_bits_to_f32(bits[:, 2 * H * D:]).astype(np.float64)
     _check(gpu, ref, float(np.sqrt(np.mean(v * v))), "full size")
+
+
+@pytest.mark.parametrize("window", [100, 64, 32768])
+def test_attention_many_short_jobs(window):
+    """Hundreds of sequences of random lengths (1 to 700 tokens) and 4 heads:
+    more jobs than the persistent grid has CTAs, so every CTA runs many jobs
+    back to back, many of them with one or two key blocks, and the pipeline's
+    barrier phases carry across job boundaries; sampled query rows of every
+    length class against the oracle."""
+    W = _W()
+    H = 4
+    rng = np.random.default_rng(window)
+    lengths = rng.integers(1, 701, size=300)
+    lengths[:8] = [1, 2, 63, 64, 65, 127, 128, 129]
+    st = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int32)
+    M = int(st[-1])
+    qkv = S.make_x(M, 3 * H * D, 300 + window, "cuda")
+    out = W.attention_prefill(qkv, torch.from_numpy(st).cuda(), H, window)
+    torch.cuda.synchronize()
+    assert W.get_device_error() == W.OK
+    # the first and last rows of every eighth sequence, and random rows
+    seq_rows = np.concatenate([[st[s], st[s + 1] - 1] for s in range(0, 300, 8)])
+    rows = np.unique(np.concatenate([seq_rows, rng.integers(0, M, size=600)])).astype(np.int64)
+    bits = S.bf16_bits(qkv)
+    ref = O.attention_rows(bits, H, D, st, window, rows=rows)
+    gpu = out[torch.from_numpy(rows).cuda()].float().cpu().numpy().astype(np.float64)
+    v = O.bf16_bits_to_f32(bits[:, 2 * H * D:]).astype(np.float64)
+    _check(gpu, ref, float(np.sqrt(np.mean(v * v))), f"many short jobs, window {window}")
