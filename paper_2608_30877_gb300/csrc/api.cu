@@ -57,6 +57,7 @@ std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 8;
+int g_gemm_cluster = 2;
 bool g_small_m_streaming = true;
 
 // Per-device set-up, done once with the device current.
@@ -81,6 +82,10 @@ int device_state(DeviceState** out) {
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
                 if (v > 0 && v <= 4096) g_group_t = v;
+            }
+            if (const char* e = std::getenv("W4A16_GEMM_CLUSTER")) {
+                if (e[0] == '1') g_gemm_cluster = 1;
+                if (e[0] == '2') g_gemm_cluster = 2;
             }
         }
         if (cudaDeviceGetAttribute(&st.sm_count, cudaDevAttrMultiProcessorCount, dev) !=
@@ -216,9 +221,11 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
+    const int cluster = v == TsVariant::kGemm256 ? g_gemm_cluster : 1;
     alignas(64) CUtensorMap tx;
     alignas(64) CUtensorMap tw;
-    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
+    // with a cluster of two, each CTA loads half of the x tile's tokens
+    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T / cluster,
                        CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != W4A16_OK) return rc;
     rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 32, 128,
@@ -236,6 +243,7 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     p.num_w_tiles = static_cast<int>((N + 127) / 128);
     p.num_tiles = p.num_t_tiles * p.num_w_tiles;
     p.group_t = v == TsVariant::kGemm256 ? g_group_t : 1;
+    p.cluster = cluster;
     p.epi = epi;
     const int grid = ts_grid(v, p, st.sm_count);
     return ts_launch(v, &tx, &tw, p, grid, stream) == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;

@@ -29,6 +29,7 @@ struct TsParams {
     int num_w_tiles;         // weight tiles: ceil(N / 128)
     int num_tiles;
     int group_t;             // raster: token tiles per group
+    int cluster;             // CTAs per cluster sharing x by multicast (1 or 2; large M only)
     Epilogue epi;
 };
 
