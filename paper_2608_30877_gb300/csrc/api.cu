@@ -56,7 +56,7 @@ struct DeviceState {
 std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
-int g_group_t = 8;
+int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
 int g_gemm_cluster = 2;
 bool g_small_m_streaming = true;
 
