@@ -295,7 +295,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     const int lane = threadIdx.x & 31;
     static_assert(CL == 1 || CL == 2, "cluster size");
     constexpr uint16_t kClusterMask = (1u << CL) - 1u;
-    const int rank = CL == 2 ? static_cast<int>(blockIdx.x & 1u) : 0;  // rank in the cluster
+    const int rank = static_cast<int>(blockIdx.x % CL);  // rank in the cluster
 
     const uint32_t bars = sbase + L::BAR_OFF;
     auto full_tma = [&](int s) { return bars + 8u * s; };
@@ -592,26 +592,27 @@ constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
 
 int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemm256 ? kGemmT : kGemvT; }
 
-// Clusters of two that can be resident at once (an SM left without a partner
-// in its GPC cannot take one); cached per device.
+// Clusters of CL that can be resident at once (SMs left over in a GPC cannot
+// take one); cached per device and cluster size.
+template <int CL>
 int gemm_cluster_slots(int sm_count) {
     constexpr int kMaxDev = 64;
     static int cache[kMaxDev] = {};
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / 2;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / CL;
     if (cache[dev] > 0) return cache[dev];
     using L = Layout<kGemmT, kGemmSS, kGemmST>;
-    auto kern = w4a16_ts_kernel<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, false, 2>;
+    auto kern = w4a16_ts_kernel<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, false, CL>;
     int n = 0;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES) ==
         cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.x = CL;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(static_cast<unsigned>(sm_count & ~1));
+        cfg.gridDim = dim3(static_cast<unsigned>(sm_count / CL * CL));
         cfg.blockDim = dim3(threads_for<kGemmDQ, kGemmEP>());
         cfg.dynamicSmemBytes = L::SMEM_BYTES;
         cfg.attrs = attr;
@@ -619,7 +620,7 @@ int gemm_cluster_slots(int sm_count) {
         if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();  // a failed query leaves no sticky error for the next launch
-    if (n <= 0) n = sm_count / 2;
+    if (n <= 0) n = sm_count / CL;
     cache[dev] = n;
     return n;
 }
@@ -628,7 +629,7 @@ int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
     if (v == TsVariant::kGemm256) {
         if (p.cluster == 2) {
             const int units = p.num_t_tiles * ((p.num_w_tiles + 1) / 2);
-            const int slots = gemm_cluster_slots(sm_count);
+            const int slots = gemm_cluster_slots<2>(sm_count);
             return 2 * (units < slots ? units : slots);
         }
         return p.num_tiles < sm_count ? p.num_tiles : sm_count;
