@@ -44,10 +44,14 @@ NCU_TRAFFIC = {
     ("qkv", "ts", "7a70fafce6ae617f"): 1.217e9 + 0.2916e9,
     # small-M readout, M = 8, 12288x49152 (DRAM counters of one launch)
     ("gemv", "gemv", "aacb64e0363a16ed"): 0.31868e9 + 0.00322e9,
+    # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
+    # one 8-pair launch); scaled by pairs / 8 for the benched launch
+    ("attention", "attn", "04bc02017fef4c26"): 0.8508e9 + 0.1827e9,
 }
 
 KERNEL_FILES = {"ts": ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"),
-                "gemv": ("gemv_rows.cu", "dequant.cuh", "ptx.cuh")}
+                "gemv": ("gemv_rows.cu", "dequant.cuh", "ptx.cuh"),
+                "attn": ("attention.cu",)}
 
 
 def kernel_source_hash(kind: str = "ts") -> str:
@@ -59,9 +63,12 @@ def kernel_source_hash(kind: str = "ts") -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(config: str, m: int):
-    if config in ("topk", "attention"):
+def ncu_traffic(config: str, m: int, pairs: int = 8):
+    if config == "topk":
         return None  # no capture of the readout kernels is summarised
+    if config == "attention":
+        t = NCU_TRAFFIC.get((config, "attn", kernel_source_hash("attn")))
+        return None if t is None else t * pairs / 8  # qkv and out grow with the pairs
     if config == "gemv":
         if m > 8:  # the capture is of the M <= 8 instantiation
             return None
@@ -639,7 +646,7 @@ def main():
         achieved = wl.flops / step_s / 1e12
         peak = peaks["bf16_tflops_sustained"] if args.config == "stack" else peaks["bf16_tflops"]
         roof = {"bound": "tensor", "unit": "TFLOP/s"}
-    traffic = ncu_traffic(args.config, args.m)
+    traffic = ncu_traffic(args.config, args.m, args.pairs)
     roof.update({"achieved": achieved, "peak": peak, "frac": achieved / peak,
                  "traffic": traffic, "peak_source": peaks["source"] + (
                      " bf16_tflops_sustained" if args.config == "stack" else
