@@ -38,7 +38,10 @@
  *     cudaGetLastError to report).
  *   - The kernels bound every internal wait.  If a wait runs out (it never
  *     should) the kernel records W4A16_ERR_TIMEOUT in a device status word
- *     and finishes early; w4a16_get_device_error reports it.
+ *     and finishes early; w4a16_get_device_error reports it.  Kernels that
+ *     check device-side data (sequence tables, gather indices) record
+ *     W4A16_ERR_INVALID_ARG there.  The word keeps the first error recorded
+ *     until it is read.
  *   - Results are deterministic: the same inputs give the same bits.
  *   - Thread safety: calls from several host threads are safe; per-device
  *     state (SM count, driver entry point) is initialised once.
@@ -71,8 +74,15 @@ typedef enum {
  *   out_bf16     [M, N]   bf16, device, written in full
  * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 32 with
  * g = 128 runs the bandwidth-bound row-range streaming kernel; other small
- * M (g != 128) run the tcgen05 kernel with 32-token tiles.  All produce the
- * same result up to fp32 summation order.
+ * M (g != 128) run the tcgen05 kernel with 32-token tiles.  The tcgen05
+ * kernels multiply x by the dequantised weights wd defined above, so they
+ * differ from each other only in the fp32 summation order.  The streaming
+ * kernel factors the scale out of each group instead: it sums x * (code - 8)
+ * over the group exactly in fp32 (the codes are small integers) and adds
+ * scale * that sum, so it never rounds (code - 8) * scale to bf16.  Both
+ * stay within the same error bound of the exact product x * wd^T (fp32
+ * accumulation followed by one bf16 rounding of the output); they are not
+ * bit-identical to each other.
  */
 int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
                  void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,
@@ -155,9 +165,15 @@ int w4a16_stack_graph_launch(w4a16_stack_graph* graph, void* stream);
 int w4a16_stack_graph_destroy(w4a16_stack_graph* graph);
 
 /*
- * wd = dequant(w_packed, scales) as bf16 [N, K] (device).  The same unpack
- * and rounding as inside the GEMM, exported so that it can be compared bit
- * for bit with the definition above.
+ * wd = dequant(w_packed, scales) as bf16 [N, K] (device): the 4-bit weights
+ * of the pre-quantised model (Sec. 4.1; "mixed-precision quantization",
+ * Sec. 3.1) brought back to the precision the matmul runs in, with the
+ * format and rounding stated at the top of this file.  The same unpack and
+ * rounding as inside the tcgen05 GEMM, exported so that it can be compared
+ * bit for bit with that definition.
+ *   w_packed_u8  [N, K/2] uint8, scales_bf16 [N, K/g] bf16, device
+ *   w_bf16       [N, K] bf16, device, written in full, must not overlap the
+ *                inputs
  */
 int w4a16_dequant(const void* w_packed_u8, const void* scales_bf16, void* w_bf16,
                   int64_t N, int64_t K, int64_t g, void* stream);
@@ -232,22 +248,37 @@ int w4a16_topk_smallest(const void* scores, int score_bits, int64_t n, int64_t k
                         void* out_index_i32, void* out_score_f32, void* stream);
 
 /*
- * Synchronises `stream`, then reads and clears the device status word that
- * kernels set when a bounded wait runs out.  Returns W4A16_OK,
- * W4A16_ERR_TIMEOUT or W4A16_ERR_CUDA.
+ * Synchronises `stream`, then reads and clears the device status word.
+ * Returns W4A16_OK, the first error a kernel recorded since the last read
+ * (W4A16_ERR_TIMEOUT from a bounded wait that ran out, W4A16_ERR_INVALID_ARG
+ * from a bad sequence table or gather index), or W4A16_ERR_CUDA if the
+ * synchronisation or the copy failed.
  */
 int w4a16_get_device_error(void* stream);
 
 /*
- * Test hook for the kernels' bounded waits; the paper has no counterpart.
- * Launches one CTA on `stream` that waits on a shared-memory mbarrier nothing
- * arrives on, giving up after limit_ns nanoseconds of global time
- * (1e3 <= limit_ns <= 1e9, else W4A16_ERR_INVALID_ARG).  On giving up it
- * records W4A16_ERR_TIMEOUT in the device status word and returns -- the same
- * path the production kernels take -- so that w4a16_get_device_error reports
- * it and the context stays usable.
+ * Test hooks for the kernels' bounded waits; the paper has no counterpart.
+ *
+ * w4a16_selftest_wait_timeout launches one CTA on `stream` whose threads
+ * wait, with the kernels' own wait helpers, on a shared-memory mbarrier that
+ * nothing arrives on: one thread gives up after limit_ns nanoseconds of
+ * global time (1e3 <= limit_ns <= 1e6, else W4A16_ERR_INVALID_ARG), raises
+ * the CTA's abort flag and records W4A16_ERR_TIMEOUT; a second warp, waiting
+ * with a far longer limit, must leave through that flag.  The timeout stays
+ * in the status word only if both waits ended that way (else the kernel
+ * records W4A16_ERR_INVALID_ARG), so w4a16_get_device_error reports it and
+ * the context stays usable.
+ *
+ * w4a16_selftest_set_wait_limit sets the wait limit of the kernels launched
+ * after it, in ns (0 < limit_ns <= 4e9; 0 restores the default of 4 s; else
+ * W4A16_ERR_INVALID_ARG).  A test lowers it so that a real kernel's waits run
+ * out and the kernel takes its abort path: it records W4A16_ERR_TIMEOUT,
+ * waits for its own copies and MMAs in flight, frees its tensor memory and
+ * returns, leaving its output incomplete.  Process-wide and not meant for
+ * concurrent use with other launches.
  */
 int w4a16_selftest_wait_timeout(int64_t limit_ns, void* stream);
+int w4a16_selftest_set_wait_limit(int64_t limit_ns);
 
 /* Static text for a status code; never NULL. */
 const char* w4a16_status_string(int status);

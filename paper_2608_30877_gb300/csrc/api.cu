@@ -10,6 +10,7 @@
 #include <cstdint>
 #include <cmath>
 #include <cstdlib>
+#include <atomic>
 #include <mutex>
 #include <new>
 
@@ -20,24 +21,35 @@ namespace {
 // w4a16_get_device_error.
 __device__ int g_status_word;
 
-// One thread waits on an mbarrier that nothing arrives on, until limit_ns of
-// global time have passed, then records a timeout like the real kernels.
+// The kernels' own wait helpers on an mbarrier that nothing arrives on:
+// thread 0 of warp 0 waits alone (wait_one) with limit_ns, the whole of
+// warp 1 waits (wait_warp) with a limit far beyond it, so it can only leave
+// through the abort flag that warp 0 raises when it gives up.  The timeout
+// that wait_one records stays in the status word only if both waits failed
+// and the flag was raised; anything else overwrites it with
+// W4A16_ERR_INVALID_ARG, which the test would report.
 __global__ void selftest_wait_kernel(uint64_t limit_ns) {
     __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    __shared__ int gave_up[2];
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&bar), 1);
+        abort_flag = 0;
+        gave_up[0] = gave_up[1] = 0;
         fence_mbar_init();
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        const uint64_t t0 = global_timer_ns();
-        while (!mbar_try_wait(smem_u32(&bar), 0)) {
-            if (global_timer_ns() - t0 > limit_ns) {
-                atomicExch(&g_status_word, W4A16_ERR_TIMEOUT);
-                break;
-            }
-        }
+    const int warp = threadIdx.x >> 5;
+    if (warp == 0) {
+        if (threadIdx.x == 0 &&
+            !wait_one(smem_u32(&bar), 0, &abort_flag, &g_status_word, limit_ns))
+            gave_up[0] = 1;
+    } else if (!wait_warp(smem_u32(&bar), 0, &abort_flag, &g_status_word, 1000u * limit_ns)) {
+        if ((threadIdx.x & 31) == 0) gave_up[1] = 1;
     }
+    __syncthreads();
+    if (threadIdx.x == 0 && !(gave_up[0] && gave_up[1] && abort_flag == 1))
+        atomicExch(&g_status_word, W4A16_ERR_INVALID_ARG);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -57,8 +69,9 @@ std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
-int g_gemm_cluster = 2;
 bool g_small_m_streaming = true;
+// barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
+std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
 
 // Per-device set-up, done once with the device current.
 int device_state(DeviceState** out) {
@@ -82,10 +95,6 @@ int device_state(DeviceState** out) {
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
                 if (v > 0 && v <= 4096) g_group_t = v;
-            }
-            if (const char* e = std::getenv("W4A16_GEMM_CLUSTER")) {
-                if (e[0] == '1') g_gemm_cluster = 1;
-                if (e[0] == '2') g_gemm_cluster = 2;
             }
         }
         if (cudaDeviceGetAttribute(&st.sm_count, cudaDevAttrMultiProcessorCount, dev) !=
@@ -209,6 +218,7 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
     p.num_chunks = static_cast<int>((N + RB - 1) / RB);
     p.nt = (RB + 127) / 128;
     p.epi = epi;
+    p.wait_ns = wait_limit_ns();
     return gemv_launch(&tx, &tw, p, st.sm_count, stream) == cudaSuccess ? W4A16_OK
                                                                          : W4A16_ERR_CUDA;
 }
@@ -221,11 +231,9 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
     const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
-    const int cluster = v == TsVariant::kGemm256 ? g_gemm_cluster : 1;
     alignas(64) CUtensorMap tx;
     alignas(64) CUtensorMap tw;
-    // with a cluster of two, each CTA loads half of the x tile's tokens
-    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T / cluster,
+    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
                        CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != W4A16_OK) return rc;
     rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 32, 128,
@@ -243,13 +251,16 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     p.num_w_tiles = static_cast<int>((N + 127) / 128);
     p.num_tiles = p.num_t_tiles * p.num_w_tiles;
     p.group_t = v == TsVariant::kGemm256 ? g_group_t : 1;
-    p.cluster = cluster;
     p.epi = epi;
+    p.wait_ns = wait_limit_ns();
     const int grid = ts_grid(v, p, st.sm_count);
     return ts_launch(v, &tx, &tw, p, grid, stream) == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
 }  // namespace
+
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
 }  // namespace w4a16
 
 using namespace w4a16;
@@ -449,6 +460,7 @@ extern "C" int w4a16_attention_prefill(const void* qkv_bf16, const void* seq_sta
     p.nseq = static_cast<int>(nseq);
     p.window = window > kMaxDim ? static_cast<int>(kMaxDim) : static_cast<int>(window);
     p.scale = 1.0f / sqrtf(static_cast<float>(d));
+    p.wait_ns = wait_limit_ns();
     return launch_attention_prefill(&tq, &tkv, p, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? W4A16_OK
                : W4A16_ERR_CUDA;
@@ -517,13 +529,23 @@ extern "C" int w4a16_get_device_error(void* stream) {
 }
 
 extern "C" int w4a16_selftest_wait_timeout(int64_t limit_ns, void* stream) {
-    if (limit_ns < 1000 || limit_ns > 1000000000) return W4A16_ERR_INVALID_ARG;
+    if (limit_ns < 1000 || limit_ns > 1000000) return W4A16_ERR_INVALID_ARG;
     DeviceState* st = nullptr;
     const int rc = device_state(&st);
     if (rc != W4A16_OK) return rc;
-    selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+    selftest_wait_kernel<<<1, 64, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<uint64_t>(limit_ns));
     return cudaGetLastError() == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
+}
+
+extern "C" int w4a16_selftest_set_wait_limit(int64_t limit_ns) {
+    if (limit_ns == 0) {
+        g_wait_limit_ns.store(kWaitLimitNs);
+        return W4A16_OK;
+    }
+    if (limit_ns < 0 || limit_ns > static_cast<int64_t>(kWaitLimitNs)) return W4A16_ERR_INVALID_ARG;
+    g_wait_limit_ns.store(static_cast<uint64_t>(limit_ns));
+    return W4A16_OK;
 }
 
 extern "C" const char* w4a16_status_string(int status) {

@@ -295,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         bad = __any_sync(0xffffffffu, bad);
         if (lane == 0) {
-            if (bad) atomicExch(p.status, 1 /* W4A16_ERR_INVALID_ARG */);
+            if (bad) record_status(p.status, 1 /* W4A16_ERR_INVALID_ARG */);
             *bad_flag = bad;
             mbar_init(q_full, 1);
             mbar_init(q_empty, 1);
@@ -337,25 +337,26 @@ __global__ void __launch_bounds__(kThreads, 2)
         // PV product is.
         bool ok = run;
         JobCursor cur;
-        uint32_t g = 0, jn = 0, nk = 0, nv = 0;
+        uint32_t g = 0, jn = 0, nq = 0, nk = 0, nv = 0;
         for (int64_t t = t_first; ok && t < njobs; t += t_step) {
             const AttnJob jb = job_at(p, t, lane, cur);
             if (!jb.valid) break;
             int b_first, nblk;
             key_range(jb, W, b_first, nblk);
             if (lane == 0) {
-                if (!wait_one(q_empty, (jn & 1u) ^ 1u, abort_flag, p.status)) ok = false;
+                if (!wait_one(q_empty, (jn & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) ok = false;
                 if (ok) {
                     mbar_arrive_expect_tx(q_full, L::Q_TILE);
                     tma_load_2d(sbase + L::Q_OFF, &tmap_q, q_full, jb.h * kD, jb.q0);
                     tma_load_2d(sbase + L::Q_OFF + L::QBOX, &tmap_q, q_full, jb.h * kD + 64, jb.q0);
+                    ++nq;
                 }
                 for (int j = 0; ok && j < nblk; ++j, ++g) {
                     const uint32_t s = g & 1u, par = ((g >> 1) & 1u) ^ 1u;
                     const int row = jb.ss + (b_first + j) * kBKV;
                     const uint32_t ks = sbase + L::K_OFF + s * L::KV_TILE;
                     const uint32_t vs = sbase + L::V_OFF + s * L::KV_TILE;
-                    if (!wait_one(k_empty(s), par, abort_flag, p.status)) {
+                    if (!wait_one(k_empty(s), par, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -363,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tma_load_2d(ks, &tmap_kv, k_full(s), Hd + jb.h * kD, row);
                     tma_load_2d(ks + L::KBOX, &tmap_kv, k_full(s), Hd + jb.h * kD + 64, row);
                     ++nk;
-                    if (!wait_one(v_empty(s), par, abort_flag, p.status)) {
+                    if (!wait_one(v_empty(s), par, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -377,14 +378,9 @@ __global__ void __launch_bounds__(kThreads, 2)
             ++jn;
         }
         if (lane == 0) {
-            // every load issued has landed before exit
-            auto settle = [&](uint32_t bar, uint32_t parity) {
-                const uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(bar, parity)) {
-                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
-                }
-            };
-            if (jn > 0) settle(q_full, (jn - 1) & 1u);
+            // every load issued has landed before exit (the Q loads are the
+            // jobs' first nq, one per job, so load i is phase i of q_full)
+            if (nq > 0) settle(q_full, (nq - 1) & 1u);
             for (uint32_t i = nk > 2 ? nk - 2 : 0; i < nk; ++i) settle(k_full(i & 1u), (i >> 1) & 1u);
             for (uint32_t i = nv > 2 ? nv - 2 : 0; i < nv; ++i) settle(v_full(i & 1u), (i >> 1) & 1u);
         }
@@ -398,8 +394,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         bool ok = run;
         auto issue_s = [&](const BlockWalk& w, uint32_t gs) -> bool {
             const uint32_t b = gs & 1u;
-            if (w.j == 0 && !wait_one(q_full, w.jn & 1u, abort_flag, p.status)) return false;
-            if (!wait_one(k_full(b), (gs >> 1) & 1u, abort_flag, p.status)) return false;
+            if (w.j == 0 && !wait_one(q_full, w.jn & 1u, abort_flag, p.status, p.wait_ns)) return false;
+            if (!wait_one(k_full(b), (gs >> 1) & 1u, abort_flag, p.status, p.wait_ns)) return false;
             tc_fence_after();
             const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + b * L::KV_TILE;
 #pragma unroll
@@ -431,8 +427,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) {
                 // O += P V once the softmax warps have written P of block g (for
                 // a job's first block, after they read out the previous job's O)
-                ok = wait_one(p_full(b), (g >> 1) & 1u, abort_flag, p.status) &&
-                     wait_one(v_full(b), (g >> 1) & 1u, abort_flag, p.status);
+                ok = wait_one(p_full(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns) &&
+                     wait_one(v_full(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns);
                 if (ok) {
                     tc_fence_after();
                     const uint32_t vs = sbase + L::V_OFF + b * L::KV_TILE;
@@ -447,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tc_commit(v_empty(b));
                 }
                 if (ok && ws.valid)
-                    ok = wait_one(o_ready(b), (g >> 1) & 1u, abort_flag, p.status) && issue_s(ws, gs);
+                    ok = wait_one(o_ready(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns) && issue_s(ws, gs);
             }
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (ws.valid) {
@@ -459,10 +455,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         if (lane == 0) {
             tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
-            const uint64_t t0 = global_timer_ns();
-            while (!mbar_try_wait(drain, 0)) {
-                if (global_timer_ns() - t0 > kWaitLimitNs) break;
-            }
+            settle(drain, 0);
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue
@@ -486,7 +479,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             float m = kMaskedScore, l = 0.0f;
             for (int j = 0; ok && j < nblk; ++j, ++g) {
                 const uint32_t b = g & 1u;
-                if (!wait_warp(s_full(b), (g >> 1) & 1u, abort_flag, p.status)) {
+                if (!wait_warp(s_full(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -560,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // rescale O (the sum over the job's blocks before j) to the new
                 // max, once the PV product of block g - 1 has completed
                 if (j > 0 && __any_sync(0xffffffffu, raise)) {
-                    if (!wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status)) {
+                    if (!wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -586,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             // ---- epilogue: O / l -> bf16.  The next job's first PV product,
             // which overwrites O, waits for P of that job, which these warps
             // write only after this epilogue has read O.
-            if (!ok || !wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status)) {
+            if (!ok || !wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
                 ok = false;
                 break;
             }
@@ -628,6 +621,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 __syncwarp();
             }
         }
+        // a softmax warp that gave up may have tensor-memory stores in flight
+        tmem_st_wait();
     }
     tc_fence_before();
     __syncthreads();

@@ -246,7 +246,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
                     const int s = it % S;
                     // a round's slots are refilled once every compute warp has left it
                     if (s % U == 0 &&
-                        !wait_one(empty(s / U), ((it / S) & 1u) ^ 1u, abort_flag, p.status)) {
+                        !wait_one(empty(s / U), ((it / S) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -267,12 +267,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
             }
             // every load this thread issued has landed before exit
             const uint32_t last = it < static_cast<uint32_t>(S) ? it : S;
-            for (uint32_t i = it - last; i < it; ++i) {
-                const uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(full(i % S), (i / S) & 1u)) {
-                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
-                }
-            }
+            for (uint32_t i = it - last; i < it; ++i) settle(full(i % S), (i / S) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ x reorder
@@ -289,7 +284,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 #pragma unroll
                 for (int u = 0; u < U; ++u) {
                     const int s = s0 + u;
-                    if (!wait_warp(full(s), ph, abort_flag, p.status)) {
+                    if (!wait_warp(full(s), ph, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -401,7 +396,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
                 const uint32_t ph = (round / RS) & 1u;
                 // ready completes after warp 1 has seen every full(s) of the
                 // round complete, so the stages' TMA data is visible here too
-                if (!wait_warp(ready(s0 / U), ph, abort_flag, p.status)) {
+                if (!wait_warp(ready(s0 / U), ph, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }

@@ -29,8 +29,8 @@ struct TsParams {
     int num_w_tiles;         // weight tiles: ceil(N / 128)
     int num_tiles;
     int group_t;             // raster: token tiles per group
-    int cluster;             // CTAs per cluster sharing x by multicast (1 or 2; large M only)
     Epilogue epi;
+    uint64_t wait_ns;        // limit of every barrier wait (kWaitLimitNs unless a test lowers it)
 };
 
 // Kernel variants of the fused kernel.  Both take 128 weight rows per tile
@@ -56,6 +56,7 @@ struct GemvParams {
     int num_chunks;          // ceil(N / RB)
     int nt;                  // MMA tiles per chunk: ceil(RB / 128)
     Epilogue epi;
+    uint64_t wait_ns;
 };
 
 // RB for N rows spread over the SMs; tokens per tile for M.
@@ -71,6 +72,7 @@ struct AttnParams {
     int* status;
     int M, H, nseq, window;
     float scale;               // 1 / sqrt(head dim)
+    uint64_t wait_ns;
 };
 int attention_head_dim();
 // tmap_q: qkv with [128 tokens x 64 features] boxes; tmap_kv: the same
@@ -87,6 +89,10 @@ cudaError_t launch_topk_smallest(const void* scores, bool bf16, int64_t n, int k
 cudaError_t launch_gather_rows(const uint16_t* src, int64_t src_rows, int64_t D,
                                const int32_t* idx, int64_t P, uint16_t* dst, int* status,
                                int sm_count, cudaStream_t stream);
+
+// Limit of the kernels' barrier waits for launches made now, in ns: 4 s
+// unless a test lowered it (w4a16_selftest_set_wait_limit).
+uint64_t wait_limit_ns();
 
 cudaError_t launch_dequant(const uint8_t* w, const uint16_t* scales, uint16_t* wd, int64_t N,
                            int64_t K, int64_t g, cudaStream_t stream);

@@ -66,24 +66,35 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Every wait in the kernels is bounded: after kWaitLimitNs of global time (or
-// kWaitIterCap polls) the waiter gives up, raises the CTA's abort flag and
-// records a timeout in the device status word.
+// Records `code` in the device status word unless an earlier error is
+// already there: the first error of a run is the one reported.
+__device__ __forceinline__ void record_status(int* status, int code) {
+    atomicCAS(status, 0, code);
+}
+
+// Every wait in the kernels is bounded: after limit_ns of global time (the
+// launch's wait limit, kWaitLimitNs unless a test lowers it) or kWaitIterCap
+// polls the waiter gives up, raises the CTA's abort flag and records a
+// timeout in the device status word.  With the default limit the clock and
+// the flag are checked every few polls; with a lowered one (a test of the
+// abort path) after every failed poll, so that the first wait that does not
+// complete at once gives up.  The drains before a kernel exits (its own
+// copies and MMAs in flight) always use kWaitLimitNs.
 constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s
 constexpr uint32_t kWaitIterCap = 1u << 26;
 
 // Wait by one thread.  Returns false if the wait ran out or the CTA aborted.
 __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status) {
+                                         int* status, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 31u) == 0u) {
+        if ((it & 31u) == 0u || limit_ns < kWaitLimitNs) {
             if (*abort_flag) return false;
-            if (it > kWaitIterCap || global_timer_ns() - t0 > kWaitLimitNs) {
+            if (it > kWaitIterCap || global_timer_ns() - t0 > limit_ns) {
                 *abort_flag = 1;
-                atomicExch(status, 5 /* W4A16_ERR_TIMEOUT */);
+                record_status(status, 5 /* W4A16_ERR_TIMEOUT */);
                 return false;
             }
         }
@@ -93,20 +104,20 @@ __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, volatile
 // Wait by a whole warp; every lane polls the barrier and the exit is
 // warp-uniform (so that .sync.aligned instructions after it stay converged).
 __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
+                                          int* status, uint64_t limit_ns) {
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
         const bool done = mbar_try_wait(bar, parity);
         if (__all_sync(0xffffffffu, done)) return true;
-        if ((it & 31u) == 31u) {
+        if ((it & 31u) == 31u || limit_ns < kWaitLimitNs) {
             int give_up = 0;
             if (lane == 0) {
                 if (*abort_flag) {
                     give_up = 1;
-                } else if (it > kWaitIterCap || global_timer_ns() - t0 > kWaitLimitNs) {
+                } else if (it > kWaitIterCap || global_timer_ns() - t0 > limit_ns) {
                     *abort_flag = 1;
-                    atomicExch(status, 5 /* W4A16_ERR_TIMEOUT */);
+                    record_status(status, 5 /* W4A16_ERR_TIMEOUT */);
                     give_up = 1;
                 }
             }
@@ -120,26 +131,36 @@ __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatil
 // issue slots from the warps doing the work.
 __device__ __forceinline__ bool wait_warp_sleep(uint32_t bar, uint32_t parity,
                                                 volatile int* abort_flag, int* status,
-                                                uint32_t sleep_ns) {
+                                                uint64_t limit_ns, uint32_t sleep_ns) {
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
         const bool done = mbar_try_wait(bar, parity);
         if (__all_sync(0xffffffffu, done)) return true;
         __nanosleep(sleep_ns);
-        if ((it & 7u) == 7u) {
+        if ((it & 7u) == 7u || limit_ns < kWaitLimitNs) {
             int give_up = 0;
             if (lane == 0) {
                 if (*abort_flag) {
                     give_up = 1;
-                } else if (it > kWaitIterCap || global_timer_ns() - t0 > kWaitLimitNs) {
+                } else if (it > kWaitIterCap || global_timer_ns() - t0 > limit_ns) {
                     *abort_flag = 1;
-                    atomicExch(status, 5 /* W4A16_ERR_TIMEOUT */);
+                    record_status(status, 5 /* W4A16_ERR_TIMEOUT */);
                     give_up = 1;
                 }
             }
             if (__shfl_sync(0xffffffffu, give_up, 0)) return false;
         }
+    }
+}
+
+// Bounded wait used by the drains before exit: gives up silently after
+// kWaitLimitNs (the copy or MMA it waits for was issued by this CTA and
+// completes on its own).
+__device__ __forceinline__ void settle(uint32_t bar, uint32_t parity) {
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_timer_ns() - t0 > kWaitLimitNs) break;
     }
 }
 
@@ -157,19 +178,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
-        : "memory");
-}
-
-// 2-D tiled load of one box, written to the same shared-memory offset in
-// every CTA of cta_mask, each of which gets the completion on its barrier at
-// offset `bar`.
-__device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst, const CUtensorMap* map,
-                                                      uint32_t bar, int32_t c0, int32_t c1,
-                                                      uint16_t cta_mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-        ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "h"(cta_mask)
         : "memory");
 }
 
@@ -233,16 +241,6 @@ __device__ __forceinline__ void tc_fence_after() {
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-        : "memory");
-}
-
-// The same arrival on the barrier at this offset in every CTA of cta_mask
-// (thread-block cluster).
-__device__ __forceinline__ void tc_commit_multicast(uint32_t bar, uint16_t cta_mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(bar),
-        "h"(cta_mask)
         : "memory");
 }
 

@@ -244,7 +244,7 @@ __global__ void gather_rows_kernel(const uint16_t* __restrict__ src, int64_t src
         uint16_t* d = dst + p * D;
         if (r < 0 || r >= src_rows) {
             for (int64_t j = threadIdx.x; j < D; j += blockDim.x) d[j] = 0;
-            if (threadIdx.x == 0) atomicExch(status, 1 /* W4A16_ERR_INVALID_ARG */);
+            if (threadIdx.x == 0) atomicCAS(status, 0, 1 /* W4A16_ERR_INVALID_ARG; the first error is kept */);
             continue;
         }
         const uint16_t* s = src + static_cast<int64_t>(r) * D;

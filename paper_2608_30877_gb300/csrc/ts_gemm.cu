@@ -28,13 +28,6 @@
 // A warp may only touch the 32 TMEM lanes of its sub-partition (warp % 4), so
 // each group of four warps covers all 128 lanes.
 //
-// Large M runs in thread-block clusters of two CTAs that take the same token
-// tile and neighbouring weight tiles in lockstep: each CTA loads half of every
-// x stage and multicasts it to both (x crosses from L2 to the SMs once per
-// two weight tiles), and a stage slot is refilled only when the MMAs of both
-// CTAs are done with it.  Under the GPU's power cap the lower on-chip traffic
-// buys clock.
-//
 // Every wait is bounded (see ptx.cuh); on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, drains its own copies and MMAs, frees tensor memory and
 // returns.
@@ -79,11 +72,11 @@ struct Layout {
     static_assert(T % 32 == 0 && T >= 32 && T <= 256, "tokens per tile");
 };
 
-// Unit -> (token tile, weight unit): units are rastered in groups of group_t
-// token tiles, token tiles fastest; a weight unit is CL consecutive weight
-// tiles (one per CTA of a cluster).
-__device__ __forceinline__ void unit_coords(int tile, const TsParams& p, int nwu, int& tt, int& wt) {
-    const int per_group = p.group_t * nwu;
+// Tile -> (token tile, weight tile): tiles are rastered in groups of group_t
+// token tiles, token tiles fastest, so that the CTAs running at the same time
+// share x and weight tiles in L2.
+__device__ __forceinline__ void tile_coords(int tile, const TsParams& p, int& tt, int& wt) {
+    const int per_group = p.group_t * p.num_w_tiles;
     const int grp = tile / per_group;
     const int first_t = grp * p.group_t;
     const int rest = p.num_t_tiles - first_t;
@@ -107,37 +100,6 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // neighbouring lanes: the even lane finishes the even tokens, the odd lane
 // the odd ones.  Otherwise neighbouring lanes swap values so that each store
 // writes the outputs (n, n+1) of one token as a 32-bit word (even n_out).
-// The units of a CTA: unit_first, + unit_stride, ... below unit_count (a
-// unit is one tile, or with clusters one token tile x CL weight tiles).
-// These read the special registers and parameters where they are used,
-// which keeps the loops' register use as low as with plain tile indices.
-template <int CL>
-__device__ __forceinline__ unsigned unit_first() { return blockIdx.x / CL; }
-template <int CL>
-__device__ __forceinline__ unsigned unit_stride() { return gridDim.x / CL; }
-template <int CL>
-__device__ __forceinline__ int weight_units(const TsParams& p) {
-    return CL == 1 ? p.num_w_tiles : (p.num_w_tiles + CL - 1) / CL;
-}
-template <int CL>
-__device__ __forceinline__ int unit_count(const TsParams& p) {
-    return CL == 1 ? p.num_tiles : p.num_t_tiles * weight_units<CL>(p);
-}
-
-// (token tile, weight tile) of rank `rank` of a cluster of CL in a unit; a
-// weight tile past N (odd tile count, second CTA) loads zeros and stores
-// nothing.
-template <int CL>
-__device__ __forceinline__ void unit_tile(int unit, const TsParams& p, int rank, int& tt, int& wt) {
-    if constexpr (CL == 1) {
-        unit_coords(unit, p, p.num_w_tiles, tt, wt);
-    } else {
-        int wu;
-        unit_coords(unit, p, weight_units<CL>(p), tt, wu);
-        wt = wu * CL + rank;
-    }
-}
-
 template <int T>
 __device__ __forceinline__ void fused_epilogue_tile(const TsParams& p, uint32_t d_col, int m0,
                                                     int n, int lane, int c0, int cs) {
@@ -275,13 +237,7 @@ constexpr int threads_for() {
     return 32 * (2 + 4 * DQ + 4 * EP);
 }
 
-// CL: CTAs per thread-block cluster.  With CL = 2 the two CTAs of a cluster
-// take the same token tile and neighbouring weight tiles in lockstep; each
-// loads half of every x stage and multicasts it to both, so x crosses from
-// L2 once per pair of weight tiles, and a stage slot is refilled only when
-// the MMAs of both CTAs are done with it (each CTA's MMA completion arrives
-// on the empty barrier of both).
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED, int CL>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED>
 __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
@@ -293,9 +249,6 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    static_assert(CL == 1 || CL == 2, "cluster size");
-    constexpr uint16_t kClusterMask = (1u << CL) - 1u;
-    const int rank = static_cast<int>(blockIdx.x % CL);  // rank in the cluster
 
     const uint32_t bars = sbase + L::BAR_OFF;
     auto full_tma = [&](int s) { return bars + 8u * s; };
@@ -311,7 +264,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     if (threadIdx.x == 0) {
         for (int s = 0; s < S_SMEM; ++s) {
             mbar_init(full_tma(s), 1);
-            mbar_init(empty_smem(s), CL);  // the MMA completion of every CTA of the cluster
+            mbar_init(empty_smem(s), 1);
         }
         for (int s = 0; s < S_TMEM; ++s) {
             mbar_init(full_a(s), 4);  // one arrival per dequant warp of the stage's group
@@ -330,10 +283,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         tmem_relinquish();
     }
     tc_fence_before();
-    if constexpr (CL > 1)
-        cluster_sync();  // barriers initialised before any peer signals them
-    else
-        __syncthreads();
+    __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
@@ -345,38 +295,27 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         if (lane == 0) {
             uint32_t it = 0;
             bool ok = true;
-            for (int unit = unit_first<CL>(); ok && unit < unit_count<CL>(p); unit += unit_stride<CL>()) {
+            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
                 int tt, wt;
-                unit_tile<CL>(unit, p, rank, tt, wt);
+                tile_coords(tile, p, tt, wt);
                 const int t0 = tt * T, n0 = wt * kRows;
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % S_SMEM;
                     const uint32_t ph = (it / S_SMEM) & 1u;
-                    if (!wait_one(empty_smem(s), ph ^ 1u, abort_flag, p.status)) {
+                    if (!wait_one(empty_smem(s), ph ^ 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
-                    // x: all of it from this CTA, or this CTA's half multicast to both
                     mbar_arrive_expect_tx(full_tma(s), L::X_BYTES + L::W_BYTES);
-                    if constexpr (CL == 1)
-                        tma_load_2d(sbase + L::X_OFF + s * L::X_BYTES, &tmap_x, full_tma(s),
-                                    kt * kBK, t0);
-                    else
-                        tma_load_2d_multicast(
-                            sbase + L::X_OFF + s * L::X_BYTES + rank * (L::X_BYTES / CL), &tmap_x,
-                            full_tma(s), kt * kBK, t0 + rank * (T / CL), kClusterMask);
+                    tma_load_2d(sbase + L::X_OFF + s * L::X_BYTES, &tmap_x, full_tma(s), kt * kBK,
+                                t0);
                     tma_load_2d(sbase + L::W_OFF + s * L::W_BYTES, &tmap_w, full_tma(s),
                                 kt * (kBK / 2), n0);
                 }
             }
             // Drain: every load this thread issued has landed before exit.
             const uint32_t last = it < static_cast<uint32_t>(S_SMEM) ? it : S_SMEM;
-            for (uint32_t i = it - last; i < it; ++i) {
-                uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(full_tma(i % S_SMEM), (i / S_SMEM) & 1u)) {
-                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
-                }
-            }
+            for (uint32_t i = it - last; i < it; ++i) settle(full_tma(i % S_SMEM), (i / S_SMEM) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -385,14 +324,14 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             uint32_t it = 0, tcount = 0;
             bool ok = true;
             bool issued = false;
-            for (int unit = unit_first<CL>(); ok && unit < unit_count<CL>(p); unit += unit_stride<CL>(), ++tcount) {
-                if (!wait_one(d_empty, (tcount & 1u) ^ 1u, abort_flag, p.status)) break;
+            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++tcount) {
+                if (!wait_one(d_empty, (tcount & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) break;
                 tc_fence_after();
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % S_SMEM;
                     const int sa = it % S_TMEM;
-                    if (!wait_one(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status) ||
-                        !wait_one(full_a(sa), (it / S_TMEM) & 1u, abort_flag, p.status)) {
+                    if (!wait_one(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status, p.wait_ns) ||
+                        !wait_one(full_a(sa), (it / S_TMEM) & 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -405,10 +344,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                         tc_mma_ts(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
                     }
                     issued = true;
-                    if constexpr (CL == 1)
-                        tc_commit(empty_smem(s));
-                    else
-                        tc_commit_multicast(empty_smem(s), kClusterMask);
+                    tc_commit(empty_smem(s));
                     tc_commit(empty_a(sa));
                 }
                 if (!ok) break;
@@ -417,21 +353,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             if (issued) {
                 // Drain: all MMAs issued by this thread have completed.
                 tc_commit(drain);
-                uint64_t t0 = global_timer_ns();
-                while (!mbar_try_wait(drain, 0)) {
-                    if (global_timer_ns() - t0 > kWaitLimitNs) break;
-                }
-            }
-            if constexpr (CL > 1) {
-                // and every CTA's completion arrivals on this CTA's empty
-                // barriers have landed (none is in flight at exit)
-                const uint32_t last = it < static_cast<uint32_t>(S_SMEM) ? it : S_SMEM;
-                for (uint32_t i = it - last; i < it; ++i) {
-                    const uint64_t t1 = global_timer_ns();
-                    while (!mbar_try_wait(empty_smem(i % S_SMEM), (i / S_SMEM) & 1u)) {
-                        if (global_timer_ns() - t1 > kWaitLimitNs) break;
-                    }
-                }
+                settle(drain, 0);
             }
         }
     } else if (warp < 2 + 4 * DQ) {
@@ -446,10 +368,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         auto grp_of = [&](int kt) { return spg_shift >= 0 ? (kt >> spg_shift) : kt / spg; };
         // scale row of the tile processed at per-CTA tile index j (nullptr: none)
         auto scale_row = [&](int j) -> const uint16_t* {
-            const int unit = unit_first<CL>() + j * unit_stride<CL>();
-            if (unit >= unit_count<CL>(p)) return nullptr;
+            const int tile = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
+            if (tile >= p.num_tiles) return nullptr;
             int tt, wt;
-            unit_tile<CL>(unit, p, rank, tt, wt);
+            tile_coords(tile, p, tt, wt);
             const int n = wt * kRows + r;
             return n < p.N ? p.scales + static_cast<int64_t>(n) * KG : nullptr;
         };
@@ -464,7 +386,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         uint32_t it = 0;
         bool ok = true;
         uint16_t s_next = load_scale(static_cast<uint32_t>(dgrp));
-        for (int j = 0, unit = unit_first<CL>(); ok && unit < unit_count<CL>(p); ++j, unit += unit_stride<CL>()) {
+        for (int j = 0, tile = blockIdx.x; ok && tile < p.num_tiles; ++j, tile += gridDim.x) {
             const uint16_t* srow = scale_row(j);
             for (int kt = 0; kt < KT; ++kt, ++it) {
                 if (static_cast<int>(it % DQ) != dgrp) continue;
@@ -476,8 +398,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     s_next = load_scale(it + DQ);
                 const int s = it % S_SMEM;
                 const int sa = it % S_TMEM;
-                if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status) ||
-                    !wait_warp(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status)) {
+                if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status, p.wait_ns) ||
+                    !wait_warp(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -511,10 +433,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const bool n_even = (p.N & 1) == 0;
         uint32_t tcount = 0;
-        for (int unit = unit_first<CL>(); unit < unit_count<CL>(p); unit += unit_stride<CL>(), ++tcount) {
+        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++tcount) {
             int tt, wt;
-            unit_tile<CL>(unit, p, rank, tt, wt);
-            if (!wait_warp_sleep(d_full, tcount & 1u, abort_flag, p.status, kEpilogueSleepNs))
+            tile_coords(tile, p, tt, wt);
+            if (!wait_warp_sleep(d_full, tcount & 1u, abort_flag, p.status, p.wait_ns, kEpilogueSleepNs))
                 break;
             tc_fence_after();
             const int n = wt * kRows + sub * 32 + lane;
@@ -529,45 +451,25 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     }
 
     tc_fence_before();
-    if constexpr (CL > 1)
-        cluster_sync();  // no CTA leaves while a peer may still signal it
-    else
-        __syncthreads();
+    __syncthreads();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, int CL>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS>
 cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
                            int grid, cudaStream_t stream) {
     using L = Layout<T, S_SMEM, S_TMEM>;
     // the plain variant carries none of the fused epilogue's code or registers
     const bool fused =
         p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
-    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true, CL>
-                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false, CL>;
+    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true>
+                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false>;
     // Idempotent; cheap enough to repeat per launch and per device.
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    if constexpr (CL == 1) {
-        kern<<<grid, threads_for<DQ, EP>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
-    } else {
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = CL;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(static_cast<unsigned>(grid));
-        cfg.blockDim = dim3(threads_for<DQ, EP>());
-        cfg.dynamicSmemBytes = L::SMEM_BYTES;
-        cfg.stream = stream;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, kern, *tx, *tw, p);
-        if (e != cudaSuccess) return e;
-    }
+    kern<<<grid, threads_for<DQ, EP>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
     return cudaGetLastError();
 }
 
@@ -592,62 +494,17 @@ constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
 
 int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemm256 ? kGemmT : kGemvT; }
 
-// Clusters of CL that can be resident at once (SMs left over in a GPC cannot
-// take one); cached per device and cluster size.
-template <int CL>
-int gemm_cluster_slots(int sm_count) {
-    constexpr int kMaxDev = 64;
-    static int cache[kMaxDev] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / CL;
-    if (cache[dev] > 0) return cache[dev];
-    using L = Layout<kGemmT, kGemmSS, kGemmST>;
-    auto kern = w4a16_ts_kernel<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, false, CL>;
-    int n = 0;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES) ==
-        cudaSuccess) {
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = CL;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(static_cast<unsigned>(sm_count / CL * CL));
-        cfg.blockDim = dim3(threads_for<kGemmDQ, kGemmEP>());
-        cfg.dynamicSmemBytes = L::SMEM_BYTES;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
-    }
-    cudaGetLastError();  // a failed query leaves no sticky error for the next launch
-    if (n <= 0) n = sm_count / CL;
-    cache[dev] = n;
-    return n;
-}
-
 int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
-    if (v == TsVariant::kGemm256) {
-        if (p.cluster == 2) {
-            const int units = p.num_t_tiles * ((p.num_w_tiles + 1) / 2);
-            const int slots = gemm_cluster_slots<2>(sm_count);
-            return 2 * (units < slots ? units : slots);
-        }
-        return p.num_tiles < sm_count ? p.num_tiles : sm_count;
-    }
+    if (v == TsVariant::kGemm256) return p.num_tiles < sm_count ? p.num_tiles : sm_count;
     return p.num_tiles;
 }
 
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
                       const TsParams& p, int grid, cudaStream_t stream) {
-    if (v == TsVariant::kGemm256) {
-        if (p.cluster == 2)
-            return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, 2>(tx, tw, p,
-                                                                                   grid, stream);
-        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, 1>(tx, tw, p, grid,
-                                                                               stream);
-    }
-    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3, 1>(tx, tw, p, grid,
-                                                                           stream);
+    if (v == TsVariant::kGemm256)
+        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1>(tx, tw, p, grid,
+                                                                            stream);
+    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3>(tx, tw, p, grid, stream);
 }
 
 }  // namespace w4a16

@@ -63,6 +63,7 @@ def lib() -> ctypes.CDLL:
         L.w4a16_quantize.argtypes = [p, p, p, i64, i64, i64, p]
         L.w4a16_get_device_error.argtypes = [p]
         L.w4a16_selftest_wait_timeout.argtypes = [i64, p]
+        L.w4a16_selftest_set_wait_limit.argtypes = [i64]
         L.w4a16_status_string.argtypes = [ctypes.c_int]
         L.w4a16_status_string.restype = ctypes.c_char_p
         L.w4a16_version.restype = ctypes.c_int
@@ -70,7 +71,8 @@ def lib() -> ctypes.CDLL:
                   "w4a16_gather_rows", "w4a16_topk_smallest", "w4a16_attention_prefill",
                   "w4a16_stack_graph_create", "w4a16_stack_graph_launch",
                   "w4a16_stack_graph_destroy", "w4a16_dequant", "w4a16_quantize",
-                  "w4a16_get_device_error", "w4a16_selftest_wait_timeout"):
+                  "w4a16_get_device_error", "w4a16_selftest_wait_timeout",
+                  "w4a16_selftest_set_wait_limit"):
             getattr(L, f).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -261,6 +263,12 @@ def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
     """Launch the bounded-wait self test (see include/w4a16.h)."""
     _check("w4a16_selftest_wait_timeout",
            lib().w4a16_selftest_wait_timeout(int(limit_ns), _stream(stream)))
+
+
+def set_wait_limit(limit_ns: int) -> None:
+    """Wait limit of the kernels launched from now on (0: the default);
+    test hook, see include/w4a16.h."""
+    _check("w4a16_selftest_set_wait_limit", lib().w4a16_selftest_set_wait_limit(int(limit_ns)))
 
 
 def get_device_error(stream=None) -> int:
