@@ -7,8 +7,8 @@ the fused epilogue swapped gate/up, a wrong SiLU sign, the tanh GELU
 approximation, a wrong residual row, bias after the activation; in the
 readout top-k ties by the last index, unordered zeros, NaN first, and a gather
 that does not zero the rows of bad indices; in attention a dropped 1/sqrt(d),
-a window one token too wide, values read from the keys, and keys of other
-sequences), points
+a window one token too wide, values read from the keys, keys of other
+sequences, and q, k, v or the output of head 0 used for every head), points
 the oracle module at it and runs the pins: at least one must fail.  The
 mistakes live only in temporary copies on the CPU."""
 import ctypes
@@ -47,6 +47,13 @@ MUTANTS = {
                                      "i - window > lo0 ? i - window : lo0")],
     "attention_v_from_k": [("qkv[j * ld + 2 * H * d + h * d + t]", "qkv[j * ld + H * d + h * d + t]")],
     "attention_ignores_sequences": [("const int64_t lo0 = seq_start[s];", "const int64_t lo0 = 0;")],
+    "attention_k_of_head_0": [("const uint16_t* k = qkv + j * ld + H * d + h * d;",
+                               "const uint16_t* k = qkv + j * ld + H * d;")],
+    "attention_q_of_head_0": [("const uint16_t* q = qkv + i * ld + h * d;",
+                               "const uint16_t* q = qkv + i * ld;")],
+    "attention_v_of_head_0": [("qkv[j * ld + 2 * H * d + h * d + t]", "qkv[j * ld + 2 * H * d + t]")],
+    "attention_out_of_head_0": [("out[r * H * d + h * d + t] = acc / den;",
+                                 "out[r * H * d + t] = acc / den;")],
     "gather_bad_rows_not_zeroed": [("for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 0;",
                                     "for (int64_t d = 0; d < D; ++d) dst[p * D + d] = 1;")],
 }
@@ -76,6 +83,7 @@ PINS = [
     P.test_attention_equal_scores_give_the_mean,
     P.test_attention_two_keys_closed_form,
     P.test_attention_is_causal_and_sequences_are_independent,
+    P.test_attention_heads_use_their_own_q_k_v_columns,
 ]
 
 

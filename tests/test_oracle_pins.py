@@ -446,3 +446,31 @@ def test_attention_is_causal_and_sequences_are_independent():
     other[:5] = O.bf16_rne_array(np.full((5, 3 * H * d), -3.0, dtype=np.float32))
     iso = O.attention_rows(other, H, d, st, window=64)
     assert np.array_equal(iso[5:], base[5:])       # another sequence does not matter
+
+
+def test_attention_heads_use_their_own_q_k_v_columns():
+    """Two heads of d = 4 (scale 1/2) whose scores differ by head: query 1 of
+    head 0 favours key 0 (scores 1, 0), query 1 of head 1 favours key 1
+    (scores 0, 2); every (token, head) has its own value vector.  Reading q,
+    k or v from another head's columns changes the weights or the values."""
+    H, d = 2, 4
+    one, two, four = 0x3F80, 0x4000, 0x4080
+    qkv = np.zeros((2, 3 * H * d), dtype=np.uint16)
+    q = lambda t, h, c, b: qkv.__setitem__((t, h * d + c), b)
+    k = lambda t, h, c, b: qkv.__setitem__((t, H * d + h * d + c), b)
+    v = lambda t, h, c, b: qkv.__setitem__((t, 2 * H * d + h * d + c), b)
+    q(1, 0, 0, two)           # head 0: q1 = 2 e0
+    q(1, 1, 1, four)          # head 1: q1 = 4 e1
+    k(0, 0, 0, one)           # head 0: k0 = e0, k1 = 0    -> scores (1, 0)
+    k(1, 1, 1, one)           # head 1: k0 = 0,  k1 = e1   -> scores (0, 2)
+    v(0, 0, 0, one)           # v of (token, head): four different unit vectors
+    v(1, 0, 1, one)
+    v(0, 1, 2, one)
+    v(1, 1, 3, one)
+    out = O.attention_rows(qkv, H, d, [0, 2], window=8)
+    e = math.e
+    want1 = np.array([e / (1 + e), 1 / (1 + e), 0, 0,
+                      0, 0, 1 / (1 + e * e), e * e / (1 + e * e)])
+    want0 = np.array([1, 0, 0, 0, 0, 0, 1, 0])   # query 0 sees only key 0
+    assert np.allclose(out[1], want1, rtol=0, atol=1e-15)
+    assert np.array_equal(out[0], want0)
