@@ -30,6 +30,36 @@ def to_device(x_bf16, packed, scales):
     return xd, wd, sd
 
 
+def prepare_weights(N, K, g, w_seed):
+    """Master weights from the generator (on the GPU), quantised on both
+    sides: the oracle's bytes are the reference (and the tensors handed to
+    the library), the library's quantiser must produce the same bytes."""
+    from paper_2608_30877_gb300 import w4a16 as W
+    master = S.make_w_master(N, K, w_seed, "cuda")
+    packed_gpu, scales_gpu = W.quantize(master, g)
+    host = master.cpu().numpy()
+    del master
+    packed, scales = O.quantize(host, g)
+    del host
+    assert np.array_equal(packed_gpu.cpu().numpy(), packed), "quantiser bytes differ"
+    assert np.array_equal(scales_gpu.cpu().view(torch.int16).numpy().view(np.uint16), scales), \
+        "quantiser scales differ"
+    return packed, scales, packed_gpu, scales_gpu
+
+
+def oracle_chain(x_bits, weights, g, nthreads=None):
+    """The oracle's own layer chain: layer i reads the bf16 rounding (the
+    oracle's RNE of the fp32 value) of the fp64 output of layer i - 1.
+    weights: [(packed, scales, N, K)]; returns the fp64 outputs per layer."""
+    nth = O.max_threads() if nthreads is None else nthreads
+    refs, xin = [], x_bits
+    for packed, scales, N, K in weights:
+        ref = O.linear_rows(xin, packed, scales, N, K, g, nthreads=nth)
+        refs.append(ref)
+        xin = O.bf16_rne_array(ref.astype(np.float32))
+    return refs
+
+
 def bf16_to_f64(t: torch.Tensor) -> np.ndarray:
     return t.detach().float().cpu().numpy().astype(np.float64)
 

@@ -13,7 +13,7 @@ import torch
 
 from oracle import oracle as O
 from paper_2608_30877_gb300 import synthetic as S
-from tests.gpu_helpers import assert_close, bf16_to_f64
+from tests.gpu_helpers import assert_close, bf16_to_f64, prepare_weights
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
@@ -34,18 +34,7 @@ def _W():
 
 
 def _prepare(N, K, g, w_seed):
-    """Master weights from the generator, quantised on both sides."""
-    W = _W()
-    master = S.make_w_master(N, K, w_seed, "cuda")
-    packed_gpu, scales_gpu = W.quantize(master, g)
-    host = master.cpu().numpy()
-    del master
-    packed, scales = O.quantize(host, g)
-    del host
-    assert np.array_equal(packed_gpu.cpu().numpy(), packed), "quantiser bytes differ"
-    assert np.array_equal(scales_gpu.cpu().view(torch.int16).numpy().view(np.uint16), scales), \
-        "quantiser scales differ"
-    return packed, scales, packed_gpu, scales_gpu
+    return prepare_weights(N, K, g, w_seed)
 
 
 def _sample_rows(M, k=6):

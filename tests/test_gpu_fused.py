@@ -8,7 +8,7 @@ import torch
 
 from oracle import oracle as O
 from paper_2608_30877_gb300 import synthetic as S
-from tests.gpu_helpers import assert_close_fused, bf16_to_f64, host_case, to_device
+from tests.gpu_helpers import assert_close_fused, bf16_to_f64, host_case, prepare_weights, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -73,3 +73,79 @@ def test_fused_none_equals_plain_linear():
     b = W.linear_fused(xd, wd, sd, g)
     torch.cuda.synchronize()
     assert torch.equal(a, b)
+
+
+def _rows(M):
+    rng = np.random.default_rng(M + 1)
+    r = {0, 255, 256, M - 1, M // 2}
+    r.update(int(v) for v in rng.integers(0, M, size=5))
+    return np.array(sorted(r), dtype=np.int64)
+
+
+@pytest.mark.slow
+def test_fused_swiglu_bias_fullsize_sampled():
+    """SwiGLU + bias on the benched gate/up shape (8192 tokens x K 12288 x
+    2 x 49152 interleaved rows): the persistent, raster-grouped GEMM over
+    many waves, on sampled token rows (all outputs) and output columns (all
+    tokens)."""
+    W = _W()
+    c = S.MLP_SWIGLU
+    packed, scales, wd, sd = prepare_weights(c.N, c.K, c.g, c.w_seed)
+    x = S.make_x(c.M, c.K, c.x_seed, "cuda")
+    rng = np.random.default_rng(11)
+    bias = S.bf16_bits(torch.from_numpy((0.5 * rng.normal(size=c.N)).astype(np.float32))
+                       .to(torch.bfloat16))
+    bias_d = torch.from_numpy(bias.view(np.int16)).view(torch.bfloat16).cuda()
+    out = W.linear_fused(x, wd, sd, c.g, act=W.ACT_SWIGLU, bias=bias_d)
+    torch.cuda.synchronize()
+    nth = O.max_threads()
+    rows = _rows(c.M)
+    ridx = torch.from_numpy(rows).cuda()
+    y = O.linear_rows(S.bf16_bits(x[ridx]), packed, scales, c.N, c.K, c.g, nthreads=nth)
+    ref = O.epilogue_rows(y, W.ACT_SWIGLU, bias=bias)
+    assert_close_fused(bf16_to_f64(out[ridx]), y, ref, W.ACT_SWIGLU, bias, "swiglu rows")
+    n_out = c.N // 2
+    cols = np.array(sorted({0, n_out // 3, n_out - 1}), dtype=np.int64)
+    wrows = np.stack([2 * cols, 2 * cols + 1], axis=1).ravel()      # (gate, up) per column
+    mi = np.repeat(np.arange(c.M, dtype=np.int64), len(wrows))
+    ni = np.tile(wrows, c.M)
+    yc = O.linear_points(S.bf16_bits(x), packed, scales, c.N, c.K, c.g, mi, ni,
+                         nthreads=nth).reshape(c.M, len(wrows))
+    refc = O.epilogue_rows(yc, W.ACT_SWIGLU, bias=bias[wrows])
+    gotc = bf16_to_f64(out[:, torch.from_numpy(cols).cuda()])
+    assert_close_fused(gotc, yc, refc, W.ACT_SWIGLU, bias[wrows], "swiglu columns")
+    assert W.get_device_error() == W.OK
+
+
+@pytest.mark.slow
+def test_fused_gelu_bias_residual_in_place_fullsize_sampled():
+    """GELU + bias + residual added in place at 8192 tokens x 12288 x 12288
+    (the persistent GEMM over many waves), on sampled rows and columns."""
+    W = _W()
+    M, N, K, g = 8192, 12288, 12288, 128
+    packed, scales, wd, sd = prepare_weights(N, K, g, 5)
+    x = S.make_x(M, K, 6, "cuda")
+    rng = np.random.default_rng(12)
+    bf = lambda a: S.bf16_bits(torch.from_numpy(a.astype(np.float32)).to(torch.bfloat16))
+    bias = bf(0.5 * rng.normal(size=N))
+    res = S.make_x(M, N, 13, "cuda")
+    res_bits = S.bf16_bits(res)
+    bias_d = torch.from_numpy(bias.view(np.int16)).view(torch.bfloat16).cuda()
+    W.linear_fused(x, wd, sd, g, act=W.ACT_GELU, bias=bias_d, residual=res, out=res)
+    torch.cuda.synchronize()
+    nth = O.max_threads()
+    rows = _rows(M)
+    ridx = torch.from_numpy(rows).cuda()
+    y = O.linear_rows(S.bf16_bits(x[ridx]), packed, scales, N, K, g, nthreads=nth)
+    ref = O.epilogue_rows(y, W.ACT_GELU, bias=bias, residual=res_bits, rows=rows)
+    assert_close_fused(bf16_to_f64(res[ridx]), y, ref, W.ACT_GELU, bias, "gelu rows")
+    cols = np.array(sorted({0, N // 3, N - 1}), dtype=np.int64)
+    mi = np.repeat(np.arange(M, dtype=np.int64), len(cols))
+    ni = np.tile(cols, M)
+    yc = O.linear_points(S.bf16_bits(x), packed, scales, N, K, g, mi, ni,
+                         nthreads=nth).reshape(M, len(cols))
+    refc = O.epilogue_rows(yc, W.ACT_GELU, bias=bias[cols],
+                           residual=np.ascontiguousarray(res_bits[:, cols]))
+    gotc = bf16_to_f64(res[:, torch.from_numpy(cols).cuda()])
+    assert_close_fused(gotc, yc, refc, W.ACT_GELU, bias[cols], "gelu columns")
+    assert W.get_device_error() == W.OK

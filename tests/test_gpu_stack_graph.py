@@ -1,12 +1,15 @@
-"""The graph-captured layer stack (w4a16_stack_graph_*) gives the same bits
-as the host-launched stack, batch after batch with new inputs copied into
-the same buffers (the continuous-batching loop), on both kernels."""
+"""The graph-captured layer stack (w4a16_stack_graph_*): batch after batch
+with new inputs copied into the same buffers (the continuous-batching loop)
+its replays give the same bits as the host-launched stack and match the
+oracle layer by layer, on both kernels and at the benched M = 65536."""
 import numpy as np
 import pytest
 import torch
 
+from oracle import oracle as O
 from paper_2608_30877_gb300 import synthetic as S
-from tests.gpu_helpers import host_case, to_device
+from tests.gpu_helpers import (assert_close, bf16_to_f64, host_case, oracle_chain,
+                               prepare_weights, to_device)
 
 pytestmark = pytest.mark.gpu
 
@@ -67,3 +70,64 @@ def test_graph_create_validates_every_layer():
         W.StackGraph([(x, w, s, out), (x, w, s, x)], M)   # second layer writes its own input
     assert e.value.status == W.ERR_INVALID_ARG
     del bad
+
+
+@pytest.mark.parametrize("M", [8, 24, 300])
+def test_graph_replay_matches_oracle_per_layer(M):
+    """Continuous batching: two batches through one captured graph; every
+    layer's output against the oracle's own layer chain on the same seeded
+    input (layer i of the chain reads the oracle's bf16 rounding of layer
+    i - 1)."""
+    W = _W()
+    K0 = 512
+    dims = [(K0, 768), (768, 512), (512, 1024), (1024, 512)]
+    xs = [torch.empty((M, K0), dtype=torch.bfloat16, device="cuda")]
+    layers, weights = [], []
+    for i, (K, N) in enumerate(dims):
+        _, _, packed, scales = host_case(1, N, K, 128, 60 + i, 61 + i)
+        _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
+        out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        layers.append((xs[-1], wd, sd, out))
+        weights.append((packed, scales, N, K))
+        xs.append(out)
+    with W.StackGraph(layers, M) as g:
+        for batch in (7, 8):
+            x0 = S.make_x(M, K0, batch, "cpu")
+            xs[0].copy_(x0.cuda())
+            g.launch()
+            torch.cuda.synchronize()
+            chain = oracle_chain(S.bf16_bits(x0), weights, 128)
+            for i, (_, _, _, out) in enumerate(layers):
+                assert_close(bf16_to_f64(out), chain[i], f"batch {batch} layer {i} M={M}")
+    assert W.get_device_error() == W.OK
+
+
+@pytest.mark.slow
+def test_graph_stack_layer0_fullsize_sampled_rows():
+    """Layer 0 of the 175B-class stack at M = 65536 (the benched launch
+    configuration), captured as a graph and replayed, against the oracle on
+    sampled token rows of each linear."""
+    W = _W()
+    M = S.STACK_M
+    layers, preps = [], []
+    for j in range(4):
+        c = S.stack_case(0, j)
+        packed, scales, wd, sd = prepare_weights(c.N, c.K, c.g, c.w_seed)
+        x = S.make_x(M, c.K, c.x_seed, "cuda")
+        out = torch.empty((M, c.N), dtype=torch.bfloat16, device="cuda")
+        layers.append((x, wd, sd, out))
+        preps.append((c, packed, scales))
+    with W.StackGraph(layers, M) as g:
+        g.launch()
+        torch.cuda.synchronize()
+    rows = np.array(sorted({0, 255, 256, 30001, M - 1}), dtype=np.int64)
+    ridx = torch.from_numpy(rows).cuda()
+    for (x, _, _, out), (c, packed, scales) in zip(layers, preps):
+        ref = O.linear_rows(S.bf16_bits(x[ridx]), packed, scales, c.N, c.K, c.g,
+                            nthreads=O.max_threads())
+        got = bf16_to_f64(out[ridx])
+        for i in range(len(rows)):
+            assert_close(got[i], ref[i], f"graph {c.name} row {rows[i]}")
+    del layers
+    torch.cuda.empty_cache()
+    assert W.get_device_error() == W.OK
