@@ -70,6 +70,7 @@ DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
 bool g_small_m_streaming = true;
+bool g_gemm_pair = false;  // large M on CTA pairs (cta_group::2)
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
 
@@ -91,6 +92,10 @@ int device_state(DeviceState** out) {
             g_encode = reinterpret_cast<EncodeTiledFn>(fn);
             if (const char* e = std::getenv("W4A16_SMALL_M_TILED")) {
                 if (e[0] == '1') g_small_m_streaming = false;
+            }
+            if (const char* e = std::getenv("W4A16_GEMM_PAIR")) {
+                if (e[0] == '1') g_gemm_pair = true;
+                if (e[0] == '0') g_gemm_pair = false;
             }
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
@@ -229,12 +234,14 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
                   cudaStream_t stream) {
     if (M <= 32 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
-    const TsVariant v = M <= 32 ? TsVariant::kGemv32 : TsVariant::kGemm256;
+    const TsVariant v = M <= 32      ? TsVariant::kGemv32
+                        : g_gemm_pair ? TsVariant::kGemmPair
+                                      : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
     alignas(64) CUtensorMap tx;
     alignas(64) CUtensorMap tw;
-    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
-                       CU_TENSOR_MAP_SWIZZLE_128B);
+    int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64,
+                       ts_x_box_tokens(v), CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != W4A16_OK) return rc;
     rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 32, 128,
                    CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -250,7 +257,7 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     p.num_t_tiles = static_cast<int>((M + T - 1) / T);
     p.num_w_tiles = static_cast<int>((N + 127) / 128);
     p.num_tiles = p.num_t_tiles * p.num_w_tiles;
-    p.group_t = v == TsVariant::kGemm256 ? g_group_t : 1;
+    p.group_t = v == TsVariant::kGemv32 ? 1 : g_group_t;
     p.epi = epi;
     p.wait_ns = wait_limit_ns();
     const int grid = ts_grid(v, p, st.sm_count);

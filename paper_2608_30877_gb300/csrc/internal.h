@@ -36,11 +36,14 @@ struct TsParams {
 // Kernel variants of the fused kernel.  Both take 128 weight rows per tile
 // (the MMA's M) and 64 k per pipeline stage.
 enum class TsVariant : int {
-    kGemm256 = 0,  // 256 tokens per tile, persistent grid (large M)
-    kGemv32 = 1,   // 32 tokens per tile, one tile per CTA (M <= 32)
+    kGemm256 = 0,   // 256 tokens per tile, persistent grid (large M)
+    kGemv32 = 1,    // 32 tokens per tile, one tile per CTA (M <= 32)
+    kGemmPair = 2,  // 256 tokens x 256 weight rows per CTA pair (cta_group::2), persistent
 };
 
 int ts_tokens_per_tile(TsVariant v);
+// Token rows of the x box each CTA loads (half the tile for CTA pairs).
+int ts_x_box_tokens(TsVariant v);
 // Fills the grid size to use for the given problem (persistent or not).
 int ts_grid(TsVariant v, const TsParams& p, int sm_count);
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,

@@ -44,9 +44,20 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
 #endif
 constexpr uint32_t kSuspendHintNs = W4A16_SUSPEND_HINT_NS;
 
+// kCluster: acquire at cluster scope, for barriers that threads or tensor-core
+// commits of the other CTA of a pair arrive on.
+template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
-    if (kSuspendHintNs == 0) {
+    if constexpr (kCluster) {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity), "r"(kSuspendHintNs == 0 ? 0x20000u : kSuspendHintNs)
+            : "memory");
+    } else if (kSuspendHintNs == 0) {
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
             "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
@@ -84,12 +95,13 @@ constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s
 constexpr uint32_t kWaitIterCap = 1u << 26;
 
 // Wait by one thread.  Returns false if the wait ran out or the CTA aborted.
+template <bool kCluster = false>
 __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                          int* status, uint64_t limit_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait<kCluster>(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait<kCluster>(bar, parity)) return true;
         if ((it & 31u) == 0u || limit_ns < kWaitLimitNs) {
             if (*abort_flag) return false;
             if (it > kWaitIterCap || global_timer_ns() - t0 > limit_ns) {
@@ -103,12 +115,13 @@ __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, volatile
 
 // Wait by a whole warp; every lane polls the barrier and the exit is
 // warp-uniform (so that .sync.aligned instructions after it stay converged).
+template <bool kCluster = false>
 __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                           int* status, uint64_t limit_ns) {
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
-        const bool done = mbar_try_wait(bar, parity);
+        const bool done = mbar_try_wait<kCluster>(bar, parity);
         if (__all_sync(0xffffffffu, done)) return true;
         if ((it & 31u) == 31u || limit_ns < kWaitLimitNs) {
             int give_up = 0;
@@ -129,13 +142,14 @@ __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatil
 // Warp-wide wait for long, latency-tolerant waits (an epilogue waiting for a
 // whole tile's MMAs): between polls the warp sleeps sleep_ns, so it takes no
 // issue slots from the warps doing the work.
+template <bool kCluster = false>
 __device__ __forceinline__ bool wait_warp_sleep(uint32_t bar, uint32_t parity,
                                                 volatile int* abort_flag, int* status,
                                                 uint64_t limit_ns, uint32_t sleep_ns) {
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
-        const bool done = mbar_try_wait(bar, parity);
+        const bool done = mbar_try_wait<kCluster>(bar, parity);
         if (__all_sync(0xffffffffu, done)) return true;
         __nanosleep(sleep_ns);
         if ((it & 7u) == 7u || limit_ns < kWaitLimitNs) {
@@ -157,9 +171,10 @@ __device__ __forceinline__ bool wait_warp_sleep(uint32_t bar, uint32_t parity,
 // Bounded wait used by the drains before exit: gives up silently after
 // kWaitLimitNs (the copy or MMA it waits for was issued by this CTA and
 // completes on its own).
+template <bool kCluster = false>
 __device__ __forceinline__ void settle(uint32_t bar, uint32_t parity) {
     const uint64_t t0 = global_timer_ns();
-    while (!mbar_try_wait(bar, parity)) {
+    while (!mbar_try_wait<kCluster>(bar, parity)) {
         if (global_timer_ns() - t0 > kWaitLimitNs) break;
     }
 }
@@ -186,6 +201,31 @@ __device__ __forceinline__ void cluster_sync() {
     asm volatile(
         "barrier.cluster.arrive.release.aligned;\n\t"
         "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Address in the shared::cluster window of the variable at shared::cta
+// address `addr` in the cluster's CTA `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// One arrival, with release at cluster scope, on an mbarrier given by its
+// shared::cluster address (this CTA's or another CTA's of the cluster).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+                 : "memory");
+}
+
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
@@ -251,6 +291,47 @@ __device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// ---- CTA pairs (cta_group::2): one MMA of M = 256 rows spans the tensor
+// cores of two CTAs of a cluster; each CTA holds its 128 rows of A and D in
+// its own tensor memory and N/2 rows of B in its own shared memory, at the
+// same addresses.  Allocation, release and deallocation are done by one warp
+// of each CTA; the MMAs and their commits by one thread of the even CTA.
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     dst_smem),
+                 "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+// Arrive once on the mbarrier at shared::cluster address `bar` (either CTA of
+// the pair) when every pair MMA issued so far by this thread has completed.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]^T over the CTA pair, kind::f16.
+__device__ __forceinline__ void tc_mma_ts_pair(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                               uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
         "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }

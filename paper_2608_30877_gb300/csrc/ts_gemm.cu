@@ -47,9 +47,12 @@ constexpr int kRows = 128;  // weight rows per tile (MMA M)
 constexpr uint32_t kEpilogueSleepNs = W4A16_EPI_SLEEP_NS;
 constexpr int kBK = 64;     // k per stage (one 128-byte swizzle row of bf16)
 
-template <int T, int S_SMEM, int S_TMEM>
+// PAIR: a CTA pair (cta_group::2) computes 2 x 128 weight rows x T tokens;
+// each CTA stages T/2 tokens of x and its own 128 weight rows.
+template <int T, int S_SMEM, int S_TMEM, bool PAIR>
 struct Layout {
-    static constexpr int X_BYTES = T * kBK * 2;
+    static constexpr int XT = PAIR ? T / 2 : T;  // tokens of x staged per CTA
+    static constexpr int X_BYTES = XT * kBK * 2;
     static constexpr int W_BYTES = kRows * kBK / 2;
     static constexpr int X_OFF = 0;
     static constexpr int W_OFF = S_SMEM * X_BYTES;
@@ -57,6 +60,8 @@ struct Layout {
     // full_tma[S_SMEM], empty_smem[S_SMEM], full_a[S_TMEM], empty_a[S_TMEM],
     // d_full, d_empty, drain
     static constexpr int NBARS = 2 * S_SMEM + 2 * S_TMEM + 3;
+    // misc: tensor-memory base, abort flag, and (pairs) the stages and tiles
+    // whose completion the MMA thread committed, handed to both CTAs at exit
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;  // + slack for 1024-B alignment
     static constexpr int D_COL = 0;
@@ -72,18 +77,45 @@ struct Layout {
     static_assert(T % 32 == 0 && T >= 32 && T <= 256, "tokens per tile");
 };
 
-// Tile -> (token tile, weight tile): tiles are rastered in groups of group_t
+// Unit -> (token tile, weight unit): units are rastered in groups of group_t
 // token tiles, token tiles fastest, so that the CTAs running at the same time
-// share x and weight tiles in L2.
-__device__ __forceinline__ void tile_coords(int tile, const TsParams& p, int& tt, int& wt) {
-    const int per_group = p.group_t * p.num_w_tiles;
-    const int grp = tile / per_group;
+// share x and weight tiles in L2.  A weight unit is CW consecutive weight
+// tiles: one per CTA (CW = 1), or the two tiles of a CTA pair (CW = 2).
+__device__ __forceinline__ void unit_coords(int unit, const TsParams& p, int nwu, int& tt, int& wu) {
+    const int per_group = p.group_t * nwu;
+    const int grp = unit / per_group;
     const int first_t = grp * p.group_t;
     const int rest = p.num_t_tiles - first_t;
     const int gsize = rest < p.group_t ? rest : p.group_t;
-    const int local = tile - grp * per_group;
+    const int local = unit - grp * per_group;
     tt = first_t + local % gsize;
-    wt = local / gsize;
+    wu = local / gsize;
+}
+
+// The units of a CTA: unit_first, + unit_stride, ... below unit_count.  The
+// two CTAs of a pair walk the same units.  These read the special registers
+// and parameters where they are used, which keeps the loops' register use as
+// low as with plain tile indices.
+template <int CW>
+__device__ __forceinline__ int unit_first() { return static_cast<int>(blockIdx.x) / CW; }
+template <int CW>
+__device__ __forceinline__ int unit_stride() { return static_cast<int>(gridDim.x) / CW; }
+template <int CW>
+__device__ __forceinline__ int weight_units(const TsParams& p) {
+    return CW == 1 ? p.num_w_tiles : (p.num_w_tiles + CW - 1) / CW;
+}
+template <int CW>
+__device__ __forceinline__ int unit_count(const TsParams& p) {
+    return CW == 1 ? p.num_tiles : p.num_t_tiles * weight_units<CW>(p);
+}
+
+// (token tile, weight tile) of the CTA of rank `rank` in its pair; a weight
+// tile past N (odd tile count, second CTA) loads zeros and stores nothing.
+template <int CW>
+__device__ __forceinline__ void unit_tile(int unit, const TsParams& p, int rank, int& tt, int& wt) {
+    int wu;
+    unit_coords(unit, p, weight_units<CW>(p), tt, wu);
+    wt = wu * CW + rank;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -237,11 +269,26 @@ constexpr int threads_for() {
     return 32 * (2 + 4 * DQ + 4 * EP);
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED>
+// PAIR = false: one CTA per tile, D[128 x T] per tcgen05.mma.cta_group::1.
+// PAIR = true: a thread-block cluster of two CTAs computes 256 weight rows x T
+// tokens with tcgen05.mma.cta_group::2 (M = 256), issued by one thread of
+// the even CTA.  Each CTA stages its own T/2 tokens of x and its own 128
+// weight rows, dequantises them into its own tensor memory (A) and holds its
+// 128 rows x T of the accumulator; the MMA reads B from both CTAs' shared
+// memory, so x crosses from L2 to the SMs once per two weight tiles and each
+// SM's shared memory supplies half of the B operand.  Hand-offs between the
+// CTAs: the odd CTA's dequant and epilogue warps arrive on the even CTA's
+// full_a and d_empty barriers (remote arrivals); the even CTA's commits
+// arrive on the empty_smem / empty_a / d_full barriers of both CTAs.  Each
+// CTA's TMA loads complete on its own full_tma barrier, which its dequant
+// warps wait on before they arrive on full_a: the MMA's wait on full_a
+// covers both CTAs' x and weight stages.
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED, bool PAIR>
 __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
-    using L = Layout<T, S_SMEM, S_TMEM>;
+    using L = Layout<T, S_SMEM, S_TMEM, PAIR>;
+    constexpr int CW = PAIR ? 2 : 1;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -249,6 +296,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;
+    const bool leader = rank == 0;  // issues the MMAs (always, without pairs)
 
     const uint32_t bars = sbase + L::BAR_OFF;
     auto full_tma = [&](int s) { return bars + 8u * s; };
@@ -260,6 +309,9 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     const uint32_t drain = d_full + 16u;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
+    volatile uint32_t* handoff = reinterpret_cast<volatile uint32_t*>(smem + L::MISC_OFF + 8);
+    // arrivals for the MMA thread go to the even CTA's barriers
+    auto at_leader = [&](uint32_t a) { return PAIR ? mapa_shared(a, 0) : a; };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S_SMEM; ++s) {
@@ -267,23 +319,33 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             mbar_init(empty_smem(s), 1);
         }
         for (int s = 0; s < S_TMEM; ++s) {
-            mbar_init(full_a(s), 4);  // one arrival per dequant warp of the stage's group
+            mbar_init(full_a(s), 4 * CW);  // one arrival per dequant warp of the stage's group, per CTA
             mbar_init(empty_a(s), 1);
         }
         mbar_init(d_full, 1);
-        mbar_init(d_empty, 4 * EP);  // one arrival per epilogue warp
+        mbar_init(d_empty, 4 * EP * CW);  // one arrival per epilogue warp, per CTA
         mbar_init(drain, 1);
         *abort_flag = 0;
+        handoff[0] = 0u;
+        handoff[1] = 0u;
         fence_mbar_init();
         prefetch_tmap(&tmap_x);
         prefetch_tmap(&tmap_w);
     }
     if (warp == 1) {
-        tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
-        tmem_relinquish();
+        if constexpr (PAIR) {
+            tmem_alloc_pair(smem_u32(tmem_slot), L::TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
-    __syncthreads();
+    if constexpr (PAIR)
+        cluster_sync();  // both CTAs' barriers and tensor memory exist before any hand-off
+    else
+        __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
@@ -295,14 +357,14 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         if (lane == 0) {
             uint32_t it = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+            for (int unit = unit_first<CW>(); ok && unit < unit_count<CW>(p); unit += unit_stride<CW>()) {
                 int tt, wt;
-                tile_coords(tile, p, tt, wt);
-                const int t0 = tt * T, n0 = wt * kRows;
+                unit_tile<CW>(unit, p, rank, tt, wt);
+                const int t0 = tt * T + rank * L::XT, n0 = wt * kRows;
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % S_SMEM;
                     const uint32_t ph = (it / S_SMEM) & 1u;
-                    if (!wait_one(empty_smem(s), ph ^ 1u, abort_flag, p.status, p.wait_ns)) {
+                    if (!wait_one<PAIR>(empty_smem(s), ph ^ 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -319,19 +381,29 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc = idesc_bf16_f32(kRows, T);
-            uint32_t it = 0, tcount = 0;
+        if (lane == 0 && leader) {
+            constexpr uint32_t idesc = idesc_bf16_f32(kRows * CW, T);
+            uint32_t it = 0, tcount = 0, tiles_done = 0;
             bool ok = true;
             bool issued = false;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++tcount) {
-                if (!wait_one(d_empty, (tcount & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) break;
+            // every commit arrives on this CTA's barrier and, for a pair, on
+            // the same barrier of the odd CTA
+            auto commit = [&](uint32_t bar) {
+                if constexpr (PAIR) {
+                    tc_commit_pair(bar);
+                    tc_commit_pair(mapa_shared(bar, 1));
+                } else {
+                    tc_commit(bar);
+                }
+            };
+            for (int unit = unit_first<CW>(); ok && unit < unit_count<CW>(p); unit += unit_stride<CW>(), ++tcount) {
+                if (!wait_one<PAIR>(d_empty, (tcount & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) break;
                 tc_fence_after();
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % S_SMEM;
                     const int sa = it % S_TMEM;
                     if (!wait_one(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status, p.wait_ns) ||
-                        !wait_one(full_a(sa), (it / S_TMEM) & 1u, abort_flag, p.status, p.wait_ns)) {
+                        !wait_one<PAIR>(full_a(sa), (it / S_TMEM) & 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -341,19 +413,34 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     for (int ks = 0; ks < kBK / 16; ++ks) {
                         const uint32_t a = tmem + L::A_COL + sa * (kBK / 2) + ks * 8;
                         const uint64_t b = sdesc_kmajor_sw128(xs + ks * 32);
-                        tc_mma_ts(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
+                        if constexpr (PAIR)
+                            tc_mma_ts_pair(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
+                        else
+                            tc_mma_ts(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
                     }
                     issued = true;
-                    tc_commit(empty_smem(s));
-                    tc_commit(empty_a(sa));
+                    commit(empty_smem(s));
+                    commit(empty_a(sa));
                 }
                 if (!ok) break;
-                tc_commit(d_full);
+                commit(d_full);
+                ++tiles_done;
             }
             if (issued) {
                 // Drain: all MMAs issued by this thread have completed.
-                tc_commit(drain);
+                if constexpr (PAIR)
+                    tc_commit_pair(drain);
+                else
+                    tc_commit(drain);
                 settle(drain, 0);
+            }
+            if constexpr (PAIR) {
+                // what both CTAs must see land on their barriers before exit
+                handoff[0] = it;
+                handoff[1] = tiles_done;
+                const uint32_t h = smem_u32(const_cast<uint32_t*>(handoff));
+                st_shared_cluster_u32(mapa_shared(h, 1), it);
+                st_shared_cluster_u32(mapa_shared(h + 4, 1), tiles_done);
             }
         }
     } else if (warp < 2 + 4 * DQ) {
@@ -366,12 +453,12 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         const int spg = p.g / kBK;
         const int spg_shift = (spg & (spg - 1)) == 0 ? __ffs(spg) - 1 : -1;
         auto grp_of = [&](int kt) { return spg_shift >= 0 ? (kt >> spg_shift) : kt / spg; };
-        // scale row of the tile processed at per-CTA tile index j (nullptr: none)
+        // scale row of the tile processed at per-CTA unit index j (nullptr: none)
         auto scale_row = [&](int j) -> const uint16_t* {
-            const int tile = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
-            if (tile >= p.num_tiles) return nullptr;
+            const int unit = unit_first<CW>() + j * unit_stride<CW>();
+            if (unit >= unit_count<CW>(p)) return nullptr;
             int tt, wt;
-            tile_coords(tile, p, tt, wt);
+            unit_tile<CW>(unit, p, rank, tt, wt);
             const int n = wt * kRows + r;
             return n < p.N ? p.scales + static_cast<int64_t>(n) * KG : nullptr;
         };
@@ -386,7 +473,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         uint32_t it = 0;
         bool ok = true;
         uint16_t s_next = load_scale(static_cast<uint32_t>(dgrp));
-        for (int j = 0, tile = blockIdx.x; ok && tile < p.num_tiles; ++j, tile += gridDim.x) {
+        for (int j = 0, unit = unit_first<CW>(); ok && unit < unit_count<CW>(p); ++j, unit += unit_stride<CW>()) {
             const uint16_t* srow = scale_row(j);
             for (int kt = 0; kt < KT; ++kt, ++it) {
                 if (static_cast<int>(it % DQ) != dgrp) continue;
@@ -399,7 +486,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 const int s = it % S_SMEM;
                 const int sa = it % S_TMEM;
                 if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status, p.wait_ns) ||
-                    !wait_warp(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
+                    !wait_warp<PAIR>(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -422,7 +509,12 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(full_a(sa));
+                if (lane == 0) {
+                    if constexpr (PAIR)
+                        mbar_arrive_cluster(at_leader(full_a(sa)));
+                    else
+                        mbar_arrive(full_a(sa));
+                }
             }
         }
     } else {
@@ -433,10 +525,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         const bool n_even = (p.N & 1) == 0;
         uint32_t tcount = 0;
-        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++tcount) {
+        for (int unit = unit_first<CW>(); unit < unit_count<CW>(p); unit += unit_stride<CW>(), ++tcount) {
             int tt, wt;
-            tile_coords(tile, p, tt, wt);
-            if (!wait_warp_sleep(d_full, tcount & 1u, abort_flag, p.status, p.wait_ns, kEpilogueSleepNs))
+            unit_tile<CW>(unit, p, rank, tt, wt);
+            if (!wait_warp_sleep<PAIR>(d_full, tcount & 1u, abort_flag, p.status, p.wait_ns, kEpilogueSleepNs))
                 break;
             tc_fence_after();
             const int n = wt * kRows + sub * 32 + lane;
@@ -446,30 +538,77 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 plain_epilogue_tile<T>(p, lane_base + L::D_COL, tt * T, n, lane, n_even, eg, EP);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(d_empty);
+            if (lane == 0) {
+                if constexpr (PAIR)
+                    mbar_arrive_cluster(at_leader(d_empty));
+                else
+                    mbar_arrive(d_empty);
+            }
         }
     }
 
+    __syncwarp();
     tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
+    if constexpr (PAIR) {
+        // Both CTAs have left their loops: no thread arrives on the other CTA
+        // any more, the MMAs have completed (drained above) and the MMA
+        // thread has handed over what it committed.  Before a CTA frees its
+        // tensor memory and exits, the commits' arrivals on its own barriers
+        // (the last stages, the last tile) must have landed.
+        cluster_sync();
+        tc_fence_after();
+        if (warp == 1) {
+            if (lane == 0) {
+                const uint32_t it = handoff[0], tiles = handoff[1];
+                const uint32_t ls = it < static_cast<uint32_t>(S_SMEM) ? it : S_SMEM;
+                for (uint32_t i = it - ls; i < it; ++i)
+                    settle<true>(empty_smem(i % S_SMEM), (i / S_SMEM) & 1u);
+                const uint32_t la = it < static_cast<uint32_t>(S_TMEM) ? it : S_TMEM;
+                for (uint32_t i = it - la; i < it; ++i)
+                    settle<true>(empty_a(i % S_TMEM), (i / S_TMEM) & 1u);
+                if (tiles > 0) settle<true>(d_full, (tiles - 1) & 1u);
+            }
+            __syncwarp();
+            tmem_dealloc_pair(tmem, L::TMEM_COLS);
+        }
+    } else {
+        __syncthreads();
+        tc_fence_after();
+        if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
+    }
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool PAIR>
 cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
                            int grid, cudaStream_t stream) {
-    using L = Layout<T, S_SMEM, S_TMEM>;
+    using L = Layout<T, S_SMEM, S_TMEM, PAIR>;
     // the plain variant carries none of the fused epilogue's code or registers
     const bool fused =
         p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
-    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true>
-                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false>;
+    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true, PAIR>
+                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false, PAIR>;
     // Idempotent; cheap enough to repeat per launch and per device.
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    kern<<<grid, threads_for<DQ, EP>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    if constexpr (!PAIR) {
+        kern<<<grid, threads_for<DQ, EP>(), L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    } else {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(static_cast<unsigned>(grid));
+        cfg.blockDim = dim3(threads_for<DQ, EP>());
+        cfg.dynamicSmemBytes = L::SMEM_BYTES;
+        cfg.stream = stream;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, kern, *tx, *tw, p);
+        if (e != cudaSuccess) return e;
+    }
     return cudaGetLastError();
 }
 
@@ -486,25 +625,76 @@ cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const T
 #endif
 constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ,
               kGemmEP = W4A16_GEMM_EP;
+// CTA pairs: 256 tokens per tile, each CTA 8 stages of (16 KB x + 4 KB packed
+// weights), the same tensor-memory split as above.
+#ifndef W4A16_PAIR_SS
+#define W4A16_PAIR_SS 8
+#endif
+constexpr int kPairSS = W4A16_PAIR_SS;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
 constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
 
+// CTA pairs that can be resident at once (SMs left over in a GPC cannot
+// take one); cached per device.
+int pair_slots(int sm_count) {
+    constexpr int kMaxDev = 64;
+    static int cache[kMaxDev] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / 2;
+    if (cache[dev] > 0) return cache[dev];
+    using L = Layout<kGemmT, kPairSS, kGemmST, true>;
+    auto kern = w4a16_ts_kernel<kGemmT, kPairSS, kGemmST, kGemmDQ, kGemmEP, 1, false, true>;
+    int n = 0;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES) ==
+        cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(static_cast<unsigned>(sm_count / 2 * 2));
+        cfg.blockDim = dim3(threads_for<kGemmDQ, kGemmEP>());
+        cfg.dynamicSmemBytes = L::SMEM_BYTES;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();  // a failed query leaves no sticky error for the next launch
+    if (n <= 0) n = sm_count / 2;
+    cache[dev] = n;
+    return n;
+}
+
 }  // namespace
 
-int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemm256 ? kGemmT : kGemvT; }
+int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemv32 ? kGemvT : kGemmT; }
+
+int ts_x_box_tokens(TsVariant v) {
+    return v == TsVariant::kGemmPair ? kGemmT / 2 : ts_tokens_per_tile(v);
+}
 
 int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
     if (v == TsVariant::kGemm256) return p.num_tiles < sm_count ? p.num_tiles : sm_count;
+    if (v == TsVariant::kGemmPair) {
+        const int units = p.num_t_tiles * ((p.num_w_tiles + 1) / 2);
+        const int slots = pair_slots(sm_count);
+        return 2 * (units < slots ? units : slots);
+    }
     return p.num_tiles;
 }
 
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
                       const TsParams& p, int grid, cudaStream_t stream) {
     if (v == TsVariant::kGemm256)
-        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1>(tx, tw, p, grid,
-                                                                            stream);
-    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3>(tx, tw, p, grid, stream);
+        return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, false>(tx, tw, p,
+                                                                                   grid, stream);
+    if (v == TsVariant::kGemmPair)
+        return launch_variant<kGemmT, kPairSS, kGemmST, kGemmDQ, kGemmEP, 1, true>(tx, tw, p,
+                                                                                  grid, stream);
+    return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3, false>(tx, tw, p, grid,
+                                                                               stream);
 }
 
 }  // namespace w4a16

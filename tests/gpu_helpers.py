@@ -72,6 +72,20 @@ def assert_close(gpu: np.ndarray, ref: np.ndarray, what: str = ""):
     return m
 
 
+def assert_close_chain(gpu: np.ndarray, ref: np.ndarray, depth: int, what: str = ""):
+    """Layer `depth` (0-based) of a chained stack against the oracle's own
+    chain.  Each layer adds its own error (the single-layer bounds) to the
+    error of its input, and a layer of random N(0, 0.02) weights maps a
+    relative input perturbation to about the same relative output
+    perturbation, so the relative errors add: the bounds are the
+    single-layer ones times depth + 1."""
+    m = O.error_metrics(gpu, ref)
+    assert np.isfinite(gpu).all(), f"{what}: non-finite output"
+    assert m["max_err_over_rms"] <= MAX_ERR_OVER_RMS * (depth + 1), f"{what}: {m}"
+    assert m["rel_fro"] <= REL_FRO * (depth + 1), f"{what}: {m}"
+    return m
+
+
 def assert_close_fused(gpu: np.ndarray, y: np.ndarray, ref: np.ndarray, act: int,
                        bias=None, what: str = ""):
     """Tolerance for fused-epilogue outputs h = act(y + bias) + residual.

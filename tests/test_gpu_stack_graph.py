@@ -8,8 +8,8 @@ import torch
 
 from oracle import oracle as O
 from paper_2608_30877_gb300 import synthetic as S
-from tests.gpu_helpers import (assert_close, bf16_to_f64, host_case, oracle_chain,
-                               prepare_weights, to_device)
+from tests.gpu_helpers import (assert_close, assert_close_chain, bf16_to_f64, host_case,
+                               oracle_chain, prepare_weights, to_device)
 
 pytestmark = pytest.mark.gpu
 
@@ -74,31 +74,59 @@ def test_graph_create_validates_every_layer():
 
 @pytest.mark.parametrize("M", [8, 24, 300])
 def test_graph_replay_matches_oracle_per_layer(M):
-    """Continuous batching: two batches through one captured graph; every
-    layer's output against the oracle's own layer chain on the same seeded
-    input (layer i of the chain reads the oracle's bf16 rounding of layer
-    i - 1)."""
+    """Continuous batching as the benchmark runs it: every layer reads its own
+    seeded input buffer; two batches (new inputs copied into the same
+    buffers) through one captured graph, every layer's output against the
+    oracle on the same seeded inputs."""
+    W = _W()
+    dims = [(512, 768), (768, 512), (512, 1024), (1024, 512)]
+    layers, weights = [], []
+    for i, (K, N) in enumerate(dims):
+        _, _, packed, scales = host_case(1, N, K, 128, 60 + i, 61 + i)
+        _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
+        x = torch.empty((M, K), dtype=torch.bfloat16, device="cuda")
+        out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        layers.append((x, wd, sd, out))
+        weights.append((packed, scales, N, K))
+    with W.StackGraph(layers, M) as g:
+        for batch in (7, 8):
+            xh = []
+            for i, (x, _, _, _) in enumerate(layers):
+                xh.append(S.make_x(M, x.shape[1], 100 * batch + i, "cpu"))
+                x.copy_(xh[-1].cuda())
+            g.launch()
+            torch.cuda.synchronize()
+            for i, ((_, _, _, out), (packed, scales, N, K)) in enumerate(zip(layers, weights)):
+                ref = O.linear_rows(S.bf16_bits(xh[i]), packed, scales, N, K, 128,
+                                    nthreads=O.max_threads())
+                assert_close(bf16_to_f64(out), ref, f"batch {batch} layer {i} M={M}")
+    assert W.get_device_error() == W.OK
+
+
+@pytest.mark.parametrize("M", [8, 300])
+def test_graph_replay_chained_matches_oracle_chain(M):
+    """A chained stack (layer i reads layer i - 1's output) replayed as a
+    graph, against the oracle's own chain on the same seeded input."""
     W = _W()
     K0 = 512
     dims = [(K0, 768), (768, 512), (512, 1024), (1024, 512)]
     xs = [torch.empty((M, K0), dtype=torch.bfloat16, device="cuda")]
     layers, weights = [], []
     for i, (K, N) in enumerate(dims):
-        _, _, packed, scales = host_case(1, N, K, 128, 60 + i, 61 + i)
+        _, _, packed, scales = host_case(1, N, K, 128, 70 + i, 71 + i)
         _, wd, sd = to_device(torch.zeros(1, K, dtype=torch.bfloat16), packed, scales)
         out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
         layers.append((xs[-1], wd, sd, out))
         weights.append((packed, scales, N, K))
         xs.append(out)
     with W.StackGraph(layers, M) as g:
-        for batch in (7, 8):
-            x0 = S.make_x(M, K0, batch, "cpu")
-            xs[0].copy_(x0.cuda())
-            g.launch()
-            torch.cuda.synchronize()
-            chain = oracle_chain(S.bf16_bits(x0), weights, 128)
-            for i, (_, _, _, out) in enumerate(layers):
-                assert_close(bf16_to_f64(out), chain[i], f"batch {batch} layer {i} M={M}")
+        x0 = S.make_x(M, K0, 9, "cpu")
+        xs[0].copy_(x0.cuda())
+        g.launch()
+        torch.cuda.synchronize()
+    chain = oracle_chain(S.bf16_bits(x0), weights, 128)
+    for i, (_, _, _, out) in enumerate(layers):
+        assert_close_chain(bf16_to_f64(out), chain[i], i, f"chained layer {i} M={M}")
     assert W.get_device_error() == W.OK
 
 
