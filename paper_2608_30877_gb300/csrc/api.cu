@@ -70,7 +70,7 @@ DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
 bool g_small_m_streaming = true;
-bool g_gemm_pair = false;  // large M on CTA pairs (cta_group::2)
+bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
 

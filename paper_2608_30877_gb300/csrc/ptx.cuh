@@ -44,18 +44,31 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
 #endif
 constexpr uint32_t kSuspendHintNs = W4A16_SUSPEND_HINT_NS;
 
+#ifndef W4A16_CLUSTER_HINT_NS
+#define W4A16_CLUSTER_HINT_NS 0x20000
+#endif
+constexpr uint32_t kClusterHintNs = W4A16_CLUSTER_HINT_NS;
+
 // kCluster: acquire at cluster scope, for barriers that threads or tensor-core
 // commits of the other CTA of a pair arrive on.
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
-    if constexpr (kCluster) {
+    if constexpr (kCluster && kClusterHintNs == 0) {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+    } else if constexpr (kCluster) {
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
             "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
             "selp.u32 %0, 1, 0, p;\n\t}"
             : "=r"(ok)
-            : "r"(bar), "r"(parity), "r"(kSuspendHintNs == 0 ? 0x20000u : kSuspendHintNs)
+            : "r"(bar), "r"(parity), "r"(kClusterHintNs)
             : "memory");
     } else if (kSuspendHintNs == 0) {
         asm volatile(
@@ -217,10 +230,14 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
     return r;
 }
 
-// One arrival, with release at cluster scope, on an mbarrier given by its
-// shared::cluster address (this CTA's or another CTA's of the cluster).
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+// One arrival without release semantics on an mbarrier of the cluster.  For
+// hand-offs of tensor-memory data only: a tcgen05.wait::st / ::ld has already
+// completed the stores or loads the arrival signals, and
+// tcgen05.fence::before_thread_sync orders them before it.  A release at
+// cluster scope here costs a cluster-wide memory fence per arrival (the CTA
+// pair GEMM ran at 916 instead of 1463 TFLOP/s with it).
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                  : "memory");
 }
 

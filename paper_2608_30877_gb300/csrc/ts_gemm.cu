@@ -278,7 +278,9 @@ constexpr int threads_for() {
 // memory, so x crosses from L2 to the SMs once per two weight tiles and each
 // SM's shared memory supplies half of the B operand.  Hand-offs between the
 // CTAs: the odd CTA's dequant and epilogue warps arrive on the even CTA's
-// full_a and d_empty barriers (remote arrivals); the even CTA's commits
+// full_a and d_empty barriers (remote arrivals without release: they hand
+// over tensor-memory reads and writes that tcgen05.wait has completed); the
+// even CTA's commits
 // arrive on the empty_smem / empty_a / d_full barriers of both CTAs.  Each
 // CTA's TMA loads complete on its own full_tma barrier, which its dequant
 // warps wait on before they arrive on full_a: the MMA's wait on full_a
@@ -289,6 +291,11 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
     using L = Layout<T, S_SMEM, S_TMEM, PAIR>;
     constexpr int CW = PAIR ? 2 : 1;
+    // Pairs run one ring: a stage's shared-memory slot and tensor-memory A
+    // slot are released together by one commit per CTA (two commits per
+    // stage instead of four; 1463 -> 1607 TFLOP/s on the QKV prefill).
+    static_assert(!PAIR || S_SMEM == S_TMEM, "pairs: one ring of stages");
+    constexpr bool kUnified = PAIR;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -420,7 +427,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     }
                     issued = true;
                     commit(empty_smem(s));
-                    commit(empty_a(sa));
+                    if constexpr (!kUnified) commit(empty_a(sa));
                 }
                 if (!ok) break;
                 commit(d_full);
@@ -486,7 +493,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 const int s = it % S_SMEM;
                 const int sa = it % S_TMEM;
                 if (!wait_warp(full_tma(s), (it / S_SMEM) & 1u, abort_flag, p.status, p.wait_ns) ||
-                    !wait_warp<PAIR>(empty_a(sa), ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
+                    !wait_warp<PAIR>(kUnified ? empty_smem(s) : empty_a(sa),
+                                     ((it / S_TMEM) & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -510,8 +518,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    if constexpr (PAIR)
-                        mbar_arrive_cluster(at_leader(full_a(sa)));
+                    // the odd CTA signals its A stage across the pair; its
+                    // tensor-memory stores are complete (wait::st above)
+                    if (PAIR && !leader)
+                        mbar_arrive_cluster_relaxed(at_leader(full_a(sa)));
                     else
                         mbar_arrive(full_a(sa));
                 }
@@ -539,8 +549,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
-                if constexpr (PAIR)
-                    mbar_arrive_cluster(at_leader(d_empty));
+                // the odd CTA's accumulator reads are complete (wait::ld in
+                // the tile's epilogue)
+                if (PAIR && !leader)
+                    mbar_arrive_cluster_relaxed(at_leader(d_empty));
                 else
                     mbar_arrive(d_empty);
             }
@@ -564,8 +576,9 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 for (uint32_t i = it - ls; i < it; ++i)
                     settle<true>(empty_smem(i % S_SMEM), (i / S_SMEM) & 1u);
                 const uint32_t la = it < static_cast<uint32_t>(S_TMEM) ? it : S_TMEM;
-                for (uint32_t i = it - la; i < it; ++i)
-                    settle<true>(empty_a(i % S_TMEM), (i / S_TMEM) & 1u);
+                if (!kUnified)
+                    for (uint32_t i = it - la; i < it; ++i)
+                        settle<true>(empty_a(i % S_TMEM), (i / S_TMEM) & 1u);
                 if (tiles > 0) settle<true>(d_full, (tiles - 1) & 1u);
             }
             __syncwarp();
@@ -625,12 +638,13 @@ cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const T
 #endif
 constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A16_GEMM_DQ,
               kGemmEP = W4A16_GEMM_EP;
-// CTA pairs: 256 tokens per tile, each CTA 8 stages of (16 KB x + 4 KB packed
-// weights), the same tensor-memory split as above.
-#ifndef W4A16_PAIR_SS
-#define W4A16_PAIR_SS 8
+// CTA pairs: 256 tokens per tile, each CTA a ring of 8 stages of (16 KB x +
+// 4 KB packed weights) and 8 tensor-memory A stages: 256 accumulator + 8 x 32
+// A columns fill the 512 columns.
+#ifndef W4A16_PAIR_STAGES
+#define W4A16_PAIR_STAGES 8
 #endif
-constexpr int kPairSS = W4A16_PAIR_SS;
+constexpr int kPairSS = W4A16_PAIR_STAGES, kPairST = W4A16_PAIR_STAGES;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
 constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
@@ -643,8 +657,8 @@ int pair_slots(int sm_count) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / 2;
     if (cache[dev] > 0) return cache[dev];
-    using L = Layout<kGemmT, kPairSS, kGemmST, true>;
-    auto kern = w4a16_ts_kernel<kGemmT, kPairSS, kGemmST, kGemmDQ, kGemmEP, 1, false, true>;
+    using L = Layout<kGemmT, kPairSS, kPairST, true>;
+    auto kern = w4a16_ts_kernel<kGemmT, kPairSS, kPairST, kGemmDQ, kGemmEP, 1, false, true>;
     int n = 0;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES) ==
         cudaSuccess) {
@@ -691,7 +705,7 @@ cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
         return launch_variant<kGemmT, kGemmSS, kGemmST, kGemmDQ, kGemmEP, 1, false>(tx, tw, p,
                                                                                    grid, stream);
     if (v == TsVariant::kGemmPair)
-        return launch_variant<kGemmT, kPairSS, kGemmST, kGemmDQ, kGemmEP, 1, true>(tx, tw, p,
+        return launch_variant<kGemmT, kPairSS, kPairST, kGemmDQ, kGemmEP, 1, true>(tx, tw, p,
                                                                                   grid, stream);
     return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3, false>(tx, tw, p, grid,
                                                                                stream);
