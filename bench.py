@@ -38,10 +38,11 @@ METRIC = "W4A16 GEMM TFLOP/s & % of roofline; scored pairs/s on 175B-class linea
 # workload and by a hash of the kernel's sources at capture time: once the
 # kernel changes the hash no longer matches and traffic is reported as null.
 NCU_TRAFFIC = {
-    # 384 launches of the timed stack step (launch list with DRAM counters)
-    ("stack", "ts", "7a70fafce6ae617f"): 30.09e9,
+    # mean of one launch per stack shape at M = 8192, scaled by 8 to M = 65536
+    # (profiles/gemm_pair_stack_traffic_m8192.md)
+    ("stack", "ts", "0e169a7ecb79efe6"): 3.67e9 * 8,
     # QKV prefill 4096x12288x36864, one launch (full capture)
-    ("qkv", "ts", "7a70fafce6ae617f"): 1.217e9 + 0.2916e9,
+    ("qkv", "ts", "0e169a7ecb79efe6"): 1.280e9 + 0.292e9,
     # small-M readout, M = 8, 12288x49152 (DRAM counters of one launch)
     ("gemv", "gemv", "aacb64e0363a16ed"): 0.31868e9 + 0.00322e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
