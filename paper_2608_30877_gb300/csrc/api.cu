@@ -70,6 +70,7 @@ DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
 bool g_small_m_streaming = true;
+bool g_small_m_tc = true;  // streaming on tcgen05; W4A16_SMALL_M=mma: the warp-level mma.sync kernel
 bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
@@ -92,6 +93,10 @@ int device_state(DeviceState** out) {
             g_encode = reinterpret_cast<EncodeTiledFn>(fn);
             if (const char* e = std::getenv("W4A16_SMALL_M_TILED")) {
                 if (e[0] == '1') g_small_m_streaming = false;
+            }
+            if (const char* e = std::getenv("W4A16_SMALL_M")) {
+                if (e[0] == 'm') g_small_m_tc = false;
+                if (e[0] == 't') g_small_m_tc = true;
             }
             if (const char* e = std::getenv("W4A16_GEMM_PAIR")) {
                 if (e[0] == '1') g_gemm_pair = true;
@@ -201,8 +206,9 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                 int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
                 cudaStream_t stream) {
-    const int T = gemv_tokens_per_tile(M);
-    const int RB = gemv_rows_per_cta(N, st.sm_count);
+    const bool tc = g_small_m_tc;
+    const int T = tc ? gemv_tc_tokens(M) : gemv_tokens_per_tile(M);
+    const int RB = tc ? gemv_tc_rows_per_cta(N, st.sm_count) : gemv_rows_per_cta(N, st.sm_count);
     alignas(64) CUtensorMap tx;
     alignas(64) CUtensorMap tw;
     int rc = encode_2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, K, M, K * 2, 64, T,
@@ -224,8 +230,9 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
     p.nt = (RB + 127) / 128;
     p.epi = epi;
     p.wait_ns = wait_limit_ns();
-    return gemv_launch(&tx, &tw, p, st.sm_count, stream) == cudaSuccess ? W4A16_OK
-                                                                         : W4A16_ERR_CUDA;
+    const cudaError_t e = tc ? gemv_tc_launch(&tx, &tw, p, st.sm_count, stream)
+                             : gemv_launch(&tx, &tw, p, st.sm_count, stream);
+    return e == cudaSuccess ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
 // Validated arguments -> one kernel launch.

@@ -118,34 +118,6 @@ __device__ __forceinline__ void mma_bf16_16816_first(float (&d)[4], uint32_t a0,
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
 }
 
-// (w >> n) & 0x000F000F | 0x43004300 as one shift and one three-input logic
-// op; written out so that the mask and the bias merge into a single LOP3.
-template <int n>
-__device__ __forceinline__ uint32_t nibble_pair_biased(uint32_t w) {
-    uint32_t r;
-    if constexpr (n == 0) {
-        asm("lop3.b32 %0, %1, 0x000F000F, 0x43004300, 0xEA;" : "=r"(r) : "r"(w));
-    } else {
-        asm("{\n\t.reg .b32 t;\n\t"
-            "shr.b32 t, %1, %2;\n\t"
-            "lop3.b32 %0, t, 0x000F000F, 0x43004300, 0xEA;\n\t}"
-            : "=r"(r)
-            : "r"(w), "n"(n));
-    }
-    return r;
-}
-
-// Codes minus the zero point, q - 8, as exact bf16 pairs (k = j, k = j + 4)
-// of one packed word: nibbles j and j + 4 sit 16 bits apart, so the mask of
-// the word shifted by 4j gives (128 + q_j, 128 + q_j+4), and subtracting 136
-// (all exact in bf16) the signed codes.
-__device__ __forceinline__ void codes_signed(uint32_t w, uint32_t* out) {
-    out[0] = bf16x2_sub(nibble_pair_biased<0>(w), 0x43084308u);
-    out[1] = bf16x2_sub(nibble_pair_biased<4>(w), 0x43084308u);
-    out[2] = bf16x2_sub(nibble_pair_biased<8>(w), 0x43084308u);
-    out[3] = bf16x2_sub(nibble_pair_biased<12>(w), 0x43084308u);
-}
-
 // Scale e of a block held as bf16 pairs, as fp32: a low half by an integer
 // multiply by 2^16 (FMA pipe), a high half by a mask.
 // (e is a constant once the stage loop is unrolled.)
@@ -159,26 +131,6 @@ __device__ __forceinline__ float scale_at(const uint32_t (&blk)[W], int e) {
     } else {
         return __uint_as_float(w & 0xFFFF0000u);
     }
-}
-
-// Shared-memory loads by 32-bit address (volatile: they stay after the
-// barrier waits that guard them).
-__device__ __forceinline__ uint2 lds64(uint32_t addr) {
-    uint2 v;
-    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint4 lds128(uint32_t addr) {
-    uint4 v;
-    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // NT: 8-token MMA column tiles (T = 8 NT staged token rows); S: stage slots;

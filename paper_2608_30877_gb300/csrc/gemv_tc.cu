@@ -1,0 +1,421 @@
+// Small-M (M <= 32, g = 128) int4-dequant + matmul on the 5th-generation
+// tensor core: the bandwidth-bound regime where the whole packed weight
+// matrix streams from HBM once per call.
+//
+// out[m, n] = sum_groups s[n, grp] * (sum_{k in grp} x[m, k] * (q[n, k] - 8)).
+//
+// Why the tensor core here: at M = 16-32 tokens the matmul is 19-39 GFLOP per
+// call, and warp-level mma.sync runs at ~610 TFLOP/s on this GPU -- 32-64 us,
+// more than the ~46 us the weights take to stream.  tcgen05.mma has four
+// times that rate and runs asynchronously, leaving the SM's integer pipes to
+// the unpacking.
+//
+// Per CTA (persistent, one per SM): a contiguous range of RB <= 384 weight
+// rows (RB = N / #SMs rounded up to even), as three MMA tiles of 128 rows.
+// Per scale group of 128 k:
+//   warp 0      TMA: two 64-k boxes of x (NTOK token rows, 128-byte swizzle,
+//               rows >= M zero-filled) and two boxes of RB/2 rows x 64 B of
+//               packed weights (64-byte swizzle) into a ring of S stages;
+//   warp 2      reorders each staged x chunk in place into the (k, k+4) pair
+//               order in which the codes come out of a packed word;
+//   warps 4-15  dequant: thread = one weight row of one tile (its TMEM lane);
+//               per 64 k, 8 words -> the exact bf16 pairs q - 8 (shift,
+//               three-input LOP3, one bf16x2 subtraction per pair; no scale
+//               multiply) -> tcgen05.st into a ring of SA A stages;
+//   warp 1      one thread issues D_grp[128 x NTOK] = A[128 x 16] x B[NTOK x 16]^T
+//               for the three tiles (A from tensor memory, B = x in shared
+//               memory), 24 MMAs per group, into one of two accumulator
+//               buffers: the group's sum of x (q - 8), exact products
+//               accumulated in fp32;
+//   warps 16-27 fold: tcgen05.ld of the group's accumulator, acc += s * D in
+//               fp32 registers (thread = row, NTOK accumulators), then the
+//               (fused) epilogue from registers.
+// The scale is applied once per group and row in fp32 (as in the warp-level
+// streaming kernel), so (q - 8) * s is never rounded to bf16; the result stays
+// within the same error bound of x * wd^T.
+//
+// Every wait is bounded (ptx.cuh); on a timeout the kernel records
+// W4A16_ERR_TIMEOUT, drains its copies and MMAs, frees tensor memory and
+// returns.
+#include "dequant.cuh"
+#include "epilogue.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace w4a16 {
+
+namespace {
+
+constexpr int kTiles = 3;                 // MMA tiles of 128 rows per CTA
+constexpr int kRowsMax = 128 * kTiles;    // rows per CTA chunk
+constexpr int kGroupK = 128;              // k per TMA stage = one scale group
+constexpr int kAK = 64;                   // k per tensor-memory A stage
+constexpr int kFirstDequantWarp = 4;      // warps 4..15 (warp % 4 = TMEM sub-partition)
+constexpr int kFirstFoldWarp = 16;        // warps 16..27
+constexpr int kRowWarps = 4 * kTiles;     // dequant (and fold) warps
+constexpr int kThreads = 32 * (kFirstFoldWarp + kRowWarps);
+
+template <int NTOK>
+struct TLayout {
+    static_assert(NTOK == 16 || NTOK == 32, "MMA N for M = 128");
+    static constexpr int S = NTOK == 32 ? 6 : 7;                     // TMA stage slots
+    static constexpr int SA = NTOK == 32 ? 3 : 4;                    // A stage slots
+    static constexpr int X_BOX = NTOK * 128;                         // 64 k x NTOK tokens
+    static constexpr int X_BYTES = 2 * X_BOX;
+    static constexpr int W_HALF = (kRowsMax / 2) * (kGroupK / 2);    // 192 rows x 64 B
+    static constexpr int W_BYTES = 2 * W_HALF;
+    static constexpr int STAGE = X_BYTES + W_BYTES;                  // x, then the weights
+    // full_tma[S], empty_smem[S], x_ready[S], full_a[SA], empty_a[SA],
+    // d_full[2], d_empty[2], drain
+    static constexpr int BAR_OFF = S * STAGE;
+    static constexpr int NBARS = 3 * S + 2 * SA + 5;
+    static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
+    static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;          // + 1024-B alignment slack
+    // tensor memory: two accumulator buffers (kTiles x NTOK columns each),
+    // then SA A stages (kTiles x 32 columns each: 64 k of bf16 pairs)
+    static constexpr int D_COLS = kTiles * NTOK;
+    static constexpr int A_COL = 2 * D_COLS;
+    static constexpr int A_COLS = kTiles * (kAK / 2);
+    static constexpr int TMEM_COLS = 512;
+    static_assert(A_COL + SA * A_COLS <= TMEM_COLS, "tensor memory holds 512 columns");
+    static_assert(X_BOX % 1024 == 0 && W_HALF % 1024 == 0 && STAGE % 1024 == 0,
+                  "swizzled boxes keep 1024-byte alignment");
+    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
+};
+
+template <int NTOK, bool FUSED>
+__global__ void __launch_bounds__(kThreads, 1)
+    w4a16_gemv_tc_kernel(const __grid_constant__ CUtensorMap tmap_x,
+                         const __grid_constant__ CUtensorMap tmap_w, const GemvParams p) {
+    using L = TLayout<NTOK>;
+    constexpr int S = L::S, SA = L::SA;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t sbase = (raw + 1023u) & ~1023u;
+    uint8_t* smem = smem_raw + (sbase - raw);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int RB = p.rows_per_cta;
+
+    const uint32_t bars = sbase + L::BAR_OFF;
+    auto full_tma = [&](int s) { return bars + 8u * s; };
+    auto empty_smem = [&](int s) { return bars + 8u * (S + s); };
+    auto x_ready = [&](int s) { return bars + 8u * (2 * S + s); };
+    auto full_a = [&](int a) { return bars + 8u * (3 * S + a); };
+    auto empty_a = [&](int a) { return bars + 8u * (3 * S + SA + a); };
+    auto d_full = [&](int b) { return bars + 8u * (3 * S + 2 * SA + b); };
+    auto d_empty = [&](int b) { return bars + 8u * (3 * S + 2 * SA + 2 + b); };
+    const uint32_t drain = bars + 8u * (3 * S + 2 * SA + 4);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_tma(s), 1);
+            mbar_init(empty_smem(s), kRowWarps + 1);  // every dequant warp read W, the MMAs read x
+            mbar_init(x_ready(s), 1);
+        }
+        for (int a = 0; a < SA; ++a) {
+            mbar_init(full_a(a), kRowWarps);
+            mbar_init(empty_a(a), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(d_full(b), 1);
+            mbar_init(d_empty(b), kRowWarps);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap_x);
+        prefetch_tmap(&tmap_w);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const int KS = p.K / kGroupK;  // scale groups = stages per chunk
+    // Each CTA walks K from its own starting group, so that the CTAs read
+    // different x slices from L2 at any moment.
+    const int rot = static_cast<int>(static_cast<int64_t>(blockIdx.x) * KS / gridDim.x);
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint32_t tx = L::X_BYTES + static_cast<uint32_t>(RB) * (kGroupK / 2);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+                const int row0 = chunk * RB;
+                int kk = rot;
+                for (int g = 0; g < KS; ++g, ++it) {
+                    const int s = it % S;
+                    if (!wait_one(empty_smem(s), ((it / S) & 1u) ^ 1u, abort_flag, p.status,
+                                  p.wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(full_tma(s), tx);
+                    const uint32_t st = sbase + s * L::STAGE;
+                    tma_load_2d(st, &tmap_x, full_tma(s), kk * kGroupK, 0);
+                    tma_load_2d(st + L::X_BOX, &tmap_x, full_tma(s), kk * kGroupK + 64, 0);
+                    tma_load_2d(st + L::X_BYTES, &tmap_w, full_tma(s), kk * (kGroupK / 2), row0);
+                    tma_load_2d(st + L::X_BYTES + L::W_HALF, &tmap_w, full_tma(s),
+                                kk * (kGroupK / 2), row0 + RB / 2);
+                    if (++kk == KS) kk = 0;
+                }
+            }
+            // every load this thread issued has landed before exit
+            const uint32_t last = it < static_cast<uint32_t>(S) ? it : S;
+            for (uint32_t i = it - last; i < it; ++i) settle(full_tma(i % S), (i / S) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_f32(128, NTOK);
+            uint32_t it = 0, ia = 0;
+            bool ok = true, issued = false;
+            for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+                for (int g = 0; ok && g < KS; ++g, ++it) {
+                    const int s = it % S;
+                    const int b = it & 1;  // accumulator buffer of this group
+                    if (!wait_one(x_ready(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns) ||
+                        !wait_one(d_empty(b), ((it >> 1) & 1u) ^ 1u, abort_flag, p.status,
+                                  p.wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t xs = sbase + s * L::STAGE;
+                    for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
+                        const int a = ia % SA;
+                        if (!wait_one(full_a(a), (ia / SA) & 1u, abort_flag, p.status, p.wait_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+#pragma unroll
+                        for (int t = 0; t < kTiles; ++t) {
+#pragma unroll
+                            for (int ks = 0; ks < kAK / 16; ++ks) {
+                                tc_mma_ts(tmem + b * L::D_COLS + t * NTOK,
+                                          tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
+                                          sdesc_kmajor_sw128(xs + h * L::X_BOX + ks * 32), idesc,
+                                          (h | ks) != 0);
+                            }
+                        }
+                        issued = true;
+                        tc_commit(empty_a(a));
+                    }
+                    if (!ok) break;
+                    tc_commit(d_full(b));
+                    tc_commit(empty_smem(s));
+                }
+            }
+            if (issued) {
+                tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
+                settle(drain, 0);
+            }
+        }
+    } else if (warp == 2) {
+        // ------------------------------------------------------------ x reorder
+        // Every 16-byte chunk (x0..x7) of the stage's x boxes becomes
+        // (x0,x4),(x1,x5),(x2,x6),(x3,x7): the pair order of codes_signed.
+        constexpr int kChunks = L::X_BYTES / 16;
+        static_assert(kChunks % 32 == 0, "whole chunks per lane");
+        uint32_t it = 0;
+        bool ok = true;
+        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+            for (int g = 0; g < KS; ++g, ++it) {
+                const int s = it % S;
+                if (!wait_warp(full_tma(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                uint4* xs = reinterpret_cast<uint4*>(smem + s * L::STAGE);
+#pragma unroll
+                for (int i = 0; i < kChunks / 32; ++i)
+                    xs[lane + 32 * i] = interleave_chunk(xs[lane + 32 * i]);
+                // these generic writes precede the MMAs' async-proxy reads
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(x_ready(s));
+            }
+        }
+    } else if (warp >= kFirstDequantWarp && warp < kFirstFoldWarp) {
+        // ------------------------------------------------------------ dequant
+        const int t = (warp - kFirstDequantWarp) >> 2;  // MMA tile
+        const int sub = warp & 3;                       // TMEM sub-partition
+        const int r = t * 128 + sub * 32 + lane;        // local row
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
+        // the row's four 16-byte chunks in a stage (64-byte swizzle)
+        const bool in_range = r < RB;
+        const int bx = r >= RB / 2 ? 1 : 0;
+        const int rr = in_range ? r - bx * (RB / 2) : 0;
+        const uint32_t row_off = L::X_BYTES + bx * L::W_HALF + rr * (kGroupK / 2);
+        const uint32_t swz = static_cast<uint32_t>((rr >> 1) & 3);
+        uint32_t it = 0, ia = 0;
+        bool ok = true;
+        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+            const bool valid = in_range && chunk * RB + r < p.N;
+            for (int g = 0; ok && g < KS; ++g, ++it) {
+                const int s = it % S;
+                if (!wait_warp(full_tma(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t wrow = sbase + s * L::STAGE + row_off;
+                for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
+                    const int a = ia % SA;
+                    uint4 c0 = make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
+                    uint4 c1 = c0;  // code 8 everywhere: rows past the range are zero
+                    if (valid) {
+                        c0 = lds128(wrow + 16u * ((2u * h) ^ swz));
+                        c1 = lds128(wrow + 16u * ((2u * h + 1u) ^ swz));
+                    }
+                    if (!wait_warp(empty_a(a), ((ia / SA) & 1u) ^ 1u, abort_flag, p.status,
+                                   p.wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint32_t v[32];
+                    codes_signed(c0.x, v + 0);
+                    codes_signed(c0.y, v + 4);
+                    codes_signed(c0.z, v + 8);
+                    codes_signed(c0.w, v + 12);
+                    codes_signed(c1.x, v + 16);
+                    codes_signed(c1.y, v + 20);
+                    codes_signed(c1.z, v + 24);
+                    codes_signed(c1.w, v + 28);
+                    tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS + t * (kAK / 2), v);
+                    tmem_st_wait();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(full_a(a));
+                }
+                if (!ok) break;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty_smem(s));  // this warp's weight reads are done
+            }
+        }
+    } else if (warp >= kFirstFoldWarp) {
+        // ------------------------------------------------------------ fold + epilogue
+        const int t = (warp - kFirstFoldWarp) >> 2;
+        const int sub = warp & 3;
+        const int r = t * 128 + sub * 32 + lane;
+        const uint32_t d_base = tmem + (static_cast<uint32_t>(sub * 32) << 16) + t * NTOK;
+        uint32_t it = 0;
+        bool ok = true;
+        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+            const int n = chunk * RB + r;
+            const bool valid = r < RB && n < p.N;
+            const uint16_t* srow = p.scales + static_cast<int64_t>(valid ? n : 0) * KS;
+            float acc[NTOK];
+#pragma unroll
+            for (int j = 0; j < NTOK; ++j) acc[j] = 0.0f;
+            int kk = rot;
+            uint16_t s_next = __ldg(srow + kk);
+            for (int g = 0; g < KS; ++g, ++it) {
+                const int b = it & 1;
+                const float sc = valid ? bf16_to_f32(s_next) : 0.0f;
+                if (++kk == KS) kk = 0;
+                if (g + 1 < KS) s_next = __ldg(srow + kk);
+                if (!wait_warp(d_full(b), (it >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+#pragma unroll
+                for (int half = 0; half < NTOK / 16; ++half) {
+                    uint32_t v[16];
+                    tmem_ld_32x32b_x16(d_base + b * L::D_COLS + half * 16, v);
+                    tmem_ld_wait_x16(v);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        acc[half * 16 + j] = fmaf(sc, __uint_as_float(v[j]), acc[half * 16 + j]);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(d_empty(b));
+            }
+            if (!ok) break;
+            // ---- epilogue from registers: row n, tokens 0 .. M - 1
+            const Epilogue& ep = p.epi;
+            if constexpr (!FUSED) {
+#pragma unroll
+                for (int m = 0; m < NTOK; ++m)
+                    if (valid && m < p.M)
+                        p.out[static_cast<int64_t>(m) * p.N + n] = f32_to_bf16_rn(acc[m]);
+            } else {
+                // SwiGLU pairs rows (n, n ^ 1) = (gate, up): RB is even, so n
+                // has the parity of its lane and the partner is lane ^ 1
+                const float bias = (ep.bias != nullptr && valid) ? bf16_to_f32(ep.bias[n]) : 0.0f;
+#pragma unroll
+                for (int m = 0; m < NTOK; ++m) {
+                    const float z = acc[m] + bias;
+                    if (ep.act == kActSwiGLU) {
+                        const float up = __shfl_xor_sync(0xffffffffu, z, 1);
+                        if ((lane & 1) == 0 && valid && m < p.M) {
+                            const int64_t o = static_cast<int64_t>(m) * ep.n_out + (n >> 1);
+                            float h = silu_f32(z) * up;
+                            if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                            p.out[o] = f32_to_bf16_rn(h);
+                        }
+                    } else if (valid && m < p.M) {
+                        const int64_t o = static_cast<int64_t>(m) * ep.n_out + n;
+                        float h = ep.act == kActGELU ? gelu_f32(z) : z;
+                        if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                        p.out[o] = f32_to_bf16_rn(h);
+                    }
+                }
+            }
+        }
+    }
+
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, L::TMEM_COLS);
+}
+
+template <int NTOK>
+cudaError_t launch_tc_variant(const CUtensorMap* tx, const CUtensorMap* tw, const GemvParams& p,
+                              int grid, cudaStream_t stream) {
+    using L = TLayout<NTOK>;
+    const bool fused =
+        p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
+    auto kern = fused ? w4a16_gemv_tc_kernel<NTOK, true> : w4a16_gemv_tc_kernel<NTOK, false>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, L::SMEM_BYTES, stream>>>(*tx, *tw, p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int gemv_tc_rows_per_cta(int64_t N, int sm_count) {
+    int64_t per = (N + sm_count - 1) / sm_count;
+    per = (per + 1) / 2 * 2;
+    if (per > kRowsMax) per = kRowsMax;
+    if (per < 2) per = 2;
+    return static_cast<int>(per);
+}
+
+int gemv_tc_tokens(int64_t M) { return M <= 16 ? 16 : 32; }
+
+cudaError_t gemv_tc_launch(const CUtensorMap* tx, const CUtensorMap* tw, const GemvParams& p,
+                           int sm_count, cudaStream_t stream) {
+    const int grid = p.num_chunks < sm_count ? p.num_chunks : sm_count;
+    if (p.M <= 16) return launch_tc_variant<16>(tx, tw, p, grid, stream);
+    return launch_tc_variant<32>(tx, tw, p, grid, stream);
+}
+
+}  // namespace w4a16

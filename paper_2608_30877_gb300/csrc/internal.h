@@ -68,6 +68,14 @@ int gemv_tokens_per_tile(int64_t M);
 cudaError_t gemv_launch(const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                         const GemvParams& p, int sm_count, cudaStream_t stream);
 
+// The tensor-core streaming kernel for the same regime (gemv_tc.cu): RB even,
+// at most 384; x boxes of gemv_tc_tokens(M) rows x 64 k (128-byte swizzle),
+// weight boxes of RB/2 rows x 64 bytes (64-byte swizzle).
+int gemv_tc_rows_per_cta(int64_t N, int sm_count);
+int gemv_tc_tokens(int64_t M);
+cudaError_t gemv_tc_launch(const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
+                           const GemvParams& p, int sm_count, cudaStream_t stream);
+
 // Attention prefill over packed sequences (attention.cu).
 struct AttnParams {
     const int32_t* seq_start;  // device [nseq + 1]
