@@ -70,7 +70,11 @@ DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
 bool g_small_m_streaming = true;
-bool g_small_m_tc = true;  // streaming on tcgen05; W4A16_SMALL_M=mma: the warp-level mma.sync kernel
+// Small M on the tcgen05 streaming kernel above this many tokens, on the
+// warp-level mma.sync kernel up to it (12288 x 49152: M = 32 108 against
+// 129 us; M = 16 104 against 85 us; M = 8 103 against 69 us).
+// W4A16_SMALL_M=mma / tc forces one of them.
+int g_small_m_tc_from = 17;
 bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
@@ -95,8 +99,8 @@ int device_state(DeviceState** out) {
                 if (e[0] == '1') g_small_m_streaming = false;
             }
             if (const char* e = std::getenv("W4A16_SMALL_M")) {
-                if (e[0] == 'm') g_small_m_tc = false;
-                if (e[0] == 't') g_small_m_tc = true;
+                if (e[0] == 'm') g_small_m_tc_from = 33;
+                if (e[0] == 't') g_small_m_tc_from = 1;
             }
             if (const char* e = std::getenv("W4A16_GEMM_PAIR")) {
                 if (e[0] == '1') g_gemm_pair = true;
@@ -206,7 +210,7 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                 int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
                 cudaStream_t stream) {
-    const bool tc = g_small_m_tc;
+    const bool tc = M >= g_small_m_tc_from;
     const int T = tc ? gemv_tc_tokens(M) : gemv_tokens_per_tile(M);
     const int RB = tc ? gemv_tc_rows_per_cta(N, st.sm_count) : gemv_rows_per_cta(N, st.sm_count);
     alignas(64) CUtensorMap tx;

@@ -22,11 +22,11 @@
 //               per 64 k, 8 words -> the exact bf16 pairs q - 8 (shift,
 //               three-input LOP3, one bf16x2 subtraction per pair; no scale
 //               multiply) -> tcgen05.st into a ring of SA A stages;
-//   warp 1      one thread issues D_grp[128 x NTOK] = A[128 x 16] x B[NTOK x 16]^T
-//               for the three tiles (A from tensor memory, B = x in shared
-//               memory), 24 MMAs per group, into one of two accumulator
-//               buffers: the group's sum of x (q - 8), exact products
-//               accumulated in fp32;
+//   warps 1, 3  one thread each, taking the groups in turn, issues
+//               D_grp[128 x NTOK] = A[128 x 16] x B[NTOK x 16]^T for the three
+//               tiles (A from tensor memory, B = x in shared memory), 24 MMAs
+//               per group, into its own accumulator buffer: the group's sum
+//               of x (q - 8), exact products accumulated in fp32;
 //   warps 16-27 fold: tcgen05.ld of the group's accumulator, acc += s * D in
 //               fp32 registers (thread = row, NTOK accumulators), then the
 //               (fused) epilogue from registers.
@@ -66,9 +66,9 @@ struct TLayout {
     static constexpr int W_BYTES = 2 * W_HALF;
     static constexpr int STAGE = X_BYTES + W_BYTES;                  // x, then the weights
     // full_tma[S], empty_smem[S], x_ready[S], full_a[SA], empty_a[SA],
-    // d_full[2], d_empty[2], drain
+    // d_full[2], d_empty[2], drain[2]
     static constexpr int BAR_OFF = S * STAGE;
-    static constexpr int NBARS = 3 * S + 2 * SA + 5;
+    static constexpr int NBARS = 3 * S + 2 * SA + 6;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;          // + 1024-B alignment slack
     // tensor memory: two accumulator buffers (kTiles x NTOK columns each),
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto empty_a = [&](int a) { return bars + 8u * (3 * S + SA + a); };
     auto d_full = [&](int b) { return bars + 8u * (3 * S + 2 * SA + b); };
     auto d_empty = [&](int b) { return bars + 8u * (3 * S + 2 * SA + 2 + b); };
-    const uint32_t drain = bars + 8u * (3 * S + 2 * SA + 4);
+    auto drain = [&](int i) { return bars + 8u * (3 * S + 2 * SA + 4 + i); };
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
 
@@ -124,7 +124,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(d_full(b), 1);
             mbar_init(d_empty(b), kRowWarps);
         }
-        mbar_init(drain, 1);
+        mbar_init(drain(0), 1);
+        mbar_init(drain(1), 1);
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tmap_x);
@@ -174,14 +175,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t last = it < static_cast<uint32_t>(S) ? it : S;
             for (uint32_t i = it - last; i < it; ++i) settle(full_tma(i % S), (i / S) & 1u);
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp == 1 || warp == 3) {
+        // ------------------------------------------------------------ MMA issuers
+        // Two threads take the groups in turn (warp 1 the even ones, with
+        // accumulator buffer 0; warp 3 the odd ones, buffer 1): one thread's
+        // commits and waits overlap the other's MMAs, and each commit tracks
+        // only its own thread's MMAs.
         if (lane == 0) {
+            const uint32_t mine = warp == 1 ? 0u : 1u;
             constexpr uint32_t idesc = idesc_bf16_f32(128, NTOK);
             uint32_t it = 0, ia = 0;
             bool ok = true, issued = false;
             for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
                 for (int g = 0; ok && g < KS; ++g, ++it) {
+                    if ((it & 1u) != mine) {
+                        ia += kGroupK / kAK;
+                        continue;
+                    }
                     const int s = it % S;
                     const int b = it & 1;  // accumulator buffer of this group
                     if (!wait_one(x_ready(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns) ||
@@ -191,7 +201,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t xs = sbase + s * L::STAGE;
+                    // descriptors and addresses of the group: one add per MMA
+                    const uint64_t bdesc = sdesc_kmajor_sw128(sbase + s * L::STAGE);
+                    const uint32_t dcol = tmem + b * L::D_COLS;
                     for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
                         const int a = ia % SA;
                         if (!wait_one(full_a(a), (ia / SA) & 1u, abort_flag, p.status, p.wait_ns)) {
@@ -199,14 +211,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                             break;
                         }
                         tc_fence_after();
+                        // consecutive MMAs go to the three tiles' accumulators in
+                        // turn, so that none waits for the one before it
 #pragma unroll
-                        for (int t = 0; t < kTiles; ++t) {
+                        for (int ks = 0; ks < kAK / 16; ++ks) {
 #pragma unroll
-                            for (int ks = 0; ks < kAK / 16; ++ks) {
-                                tc_mma_ts(tmem + b * L::D_COLS + t * NTOK,
+                            for (int t = 0; t < kTiles; ++t) {
+                                // the descriptor's start address is in 16-byte units
+                                tc_mma_ts(dcol + t * NTOK,
                                           tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
-                                          sdesc_kmajor_sw128(xs + h * L::X_BOX + ks * 32), idesc,
-                                          (h | ks) != 0);
+                                          bdesc + static_cast<uint64_t>((h * L::X_BOX + ks * 32) >> 4),
+                                          idesc, (h | ks) != 0);
                             }
                         }
                         issued = true;
@@ -218,8 +233,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (issued) {
-                tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
-                settle(drain, 0);
+                // every MMA issued has completed before tensor memory is freed
+                tc_commit(drain(mine));
+                settle(drain(mine), 0);
             }
         }
     } else if (warp == 2) {

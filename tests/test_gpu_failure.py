@@ -70,9 +70,11 @@ def short_waits():
         W.set_wait_limit(0)
 
 
-# (M, N, K, g): large-M tcgen05 GEMM (several tiles per CTA), the small-M
-# streaming kernel, the 32-token tcgen05 tiles (g = 64)
-ABORT_CASES = [(600, 128 * 400, 2048, 128), (8, 8192, 4096, 128), (16, 4096, 1024, 64)]
+# (M, N, K, g): large-M tcgen05 GEMM on CTA pairs (several tiles per pair),
+# the warp-level small-M streaming kernel, the tcgen05 small-M streaming
+# kernel, the 32-token tcgen05 tiles (g = 64)
+ABORT_CASES = [(600, 128 * 400, 2048, 128), (8, 8192, 4096, 128), (24, 8192, 4096, 128),
+               (16, 4096, 1024, 64)]
 
 
 @pytest.mark.parametrize("M,N,K,g", ABORT_CASES)

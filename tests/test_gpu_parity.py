@@ -192,3 +192,38 @@ def test_small_m_streaming_kernel_shapes(M, N, K, g):
     second row range (more row ranges than SMs)."""
     gpu, ref = _run_linear(M, N, K, g, seed=3 * M + N)
     assert_close(gpu, ref, f"{M}x{K}x{N} g{g}")
+
+
+_FORCED_KERNEL_CHECK = r"""
+import sys
+import numpy as np, torch
+sys.path.insert(0, {root!r})
+from oracle import oracle as O
+from tests.gpu_helpers import assert_close, bf16_to_f64, host_case, to_device
+from paper_2608_30877_gb300 import w4a16 as W
+for (M, N, K) in {cases!r}:
+    x, xb, packed, scales = host_case(M, N, K, 128, 300 + M, 301 + M)
+    xd, wd, sd = to_device(x, packed, scales)
+    out = W.linear(xd, wd, sd, 128)
+    torch.cuda.synchronize()
+    ref = O.linear_rows(xb, packed, scales, N, K, 128, nthreads=O.max_threads())
+    assert_close(bf16_to_f64(out), ref, f"M={{M}} N={{N}} K={{K}}")
+assert W.get_device_error() == W.OK
+print("ok")
+"""
+
+
+@pytest.mark.parametrize("kernel", ["tc", "mma"])
+def test_small_m_kernels_every_m(kernel):
+    """Both small-M streaming kernels at every M they can be forced to
+    (W4A16_SMALL_M), on ragged shapes: the dispatch picks one by M, and
+    each must be correct everywhere."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    cases = [(M, 1000 + 2 * M, 384 if M % 2 else 1280) for M in (1, 2, 5, 8, 13, 16, 17, 24, 31, 32)]
+    env = dict(os.environ, W4A16_SMALL_M=kernel)
+    r = subprocess.run([sys.executable, "-c", _FORCED_KERNEL_CHECK.format(root=root, cases=cases)],
+                       env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0 and "ok" in r.stdout, r.stdout + r.stderr
