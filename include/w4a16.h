@@ -45,6 +45,11 @@
  *   - Results are deterministic: the same inputs give the same bits.
  *   - Thread safety: calls from several host threads are safe; per-device
  *     state (SM count, driver entry point) is initialised once.
+ *   - Debug build: compiled with -DW4A16_DEBUG (libw4a16_debug.so), the
+ *     kernels check every TMA coordinate and destination, tensor-memory column
+ *     range and global store index they compute; a failed check records
+ *     W4A16_ERR_INDEX in the device status word and skips the access (no
+ *     trap).  The release build carries none of these checks.
  */
 #ifndef W4A16_H
 #define W4A16_H
@@ -61,7 +66,8 @@ typedef enum {
     W4A16_ERR_UNSUPPORTED = 2,   /* valid request outside the supported shapes */
     W4A16_ERR_ALIGNMENT = 3,     /* a pointer is not 16-byte aligned */
     W4A16_ERR_CUDA = 4,          /* a CUDA runtime/driver call or launch failed */
-    W4A16_ERR_TIMEOUT = 5        /* a kernel gave up on a bounded wait */
+    W4A16_ERR_TIMEOUT = 5,       /* a kernel gave up on a bounded wait */
+    W4A16_ERR_INDEX = 6          /* an index check of a W4A16_DEBUG build failed */
 } w4a16_status;
 
 /*

@@ -574,6 +574,7 @@ extern "C" const char* w4a16_status_string(int status) {
         case W4A16_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
         case W4A16_ERR_CUDA: return "CUDA error";
         case W4A16_ERR_TIMEOUT: return "kernel wait timed out";
+        case W4A16_ERR_INDEX: return "index check failed (debug build)";
         default: return "unknown status";
     }
 }

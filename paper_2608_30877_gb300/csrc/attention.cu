@@ -347,8 +347,16 @@ __global__ void __launch_bounds__(kThreads, 2)
                 if (!wait_one(q_empty, (jn & 1u) ^ 1u, abort_flag, p.status, p.wait_ns)) ok = false;
                 if (ok) {
                     mbar_arrive_expect_tx(q_full, L::Q_TILE);
-                    tma_load_2d(sbase + L::Q_OFF, &tmap_q, q_full, jb.h * kD, jb.q0);
-                    tma_load_2d(sbase + L::Q_OFF + L::QBOX, &tmap_q, q_full, jb.h * kD + 64, jb.q0);
+                    if (dbg_check(tma_box_ok(sbase + L::Q_OFF, L::QBOX, 1024, sbase,
+                                             sbase + L::K_OFF, jb.h * kD, 2) &&
+                                      tma_box_ok(sbase + L::Q_OFF + L::QBOX, L::QBOX, 1024, sbase,
+                                                 sbase + L::K_OFF, jb.h * kD + 64, 2) &&
+                                      jb.q0 >= 0 && jb.q0 < p.M,
+                                  p.status)) {
+                        tma_load_2d(sbase + L::Q_OFF, &tmap_q, q_full, jb.h * kD, jb.q0);
+                        tma_load_2d(sbase + L::Q_OFF + L::QBOX, &tmap_q, q_full, jb.h * kD + 64,
+                                    jb.q0);
+                    }
                     ++nq;
                 }
                 for (int j = 0; ok && j < nblk; ++j, ++g) {
@@ -361,16 +369,27 @@ __global__ void __launch_bounds__(kThreads, 2)
                         break;
                     }
                     mbar_arrive_expect_tx(k_full(s), L::KV_TILE);
-                    tma_load_2d(ks, &tmap_kv, k_full(s), Hd + jb.h * kD, row);
-                    tma_load_2d(ks + L::KBOX, &tmap_kv, k_full(s), Hd + jb.h * kD + 64, row);
+                    // key rows of the block start inside the job's sequence
+                    if (dbg_check(tma_box_ok(ks, L::KV_TILE, 1024, sbase + L::K_OFF,
+                                             sbase + L::V_OFF, Hd + jb.h * kD, 2) &&
+                                      row >= jb.ss && row < jb.se,
+                                  p.status)) {
+                        tma_load_2d(ks, &tmap_kv, k_full(s), Hd + jb.h * kD, row);
+                        tma_load_2d(ks + L::KBOX, &tmap_kv, k_full(s), Hd + jb.h * kD + 64, row);
+                    }
                     ++nk;
                     if (!wait_one(v_empty(s), par, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
                     mbar_arrive_expect_tx(v_full(s), L::KV_TILE);
-                    tma_load_2d(vs, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD, row);
-                    tma_load_2d(vs + L::KBOX, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD + 64, row);
+                    if (dbg_check(tma_box_ok(vs, L::KV_TILE, 1024, sbase + L::V_OFF,
+                                             sbase + L::STAGE_OFF, 2 * Hd + jb.h * kD, 2),
+                                  p.status)) {
+                        tma_load_2d(vs, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD, row);
+                        tma_load_2d(vs + L::KBOX, &tmap_kv, v_full(s), 2 * Hd + jb.h * kD + 64,
+                                    row);
+                    }
                     ++nv;
                 }
             }
@@ -615,7 +634,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const int q = it * 8 + (lane >> 2), u = lane & 3;
                     const uint4 w = *reinterpret_cast<const uint4*>(stage + q * 64 +
                                                                     ((u ^ ((q >> 1) & 3)) << 4));
-                    if (q < rows_left)
+                    if (q < rows_left &&
+                        dbg_check(jb.q0 + sub * 32 + q < jb.se && jb.q0 + sub * 32 + q >= jb.ss,
+                                  p.status))
                         *reinterpret_cast<uint4*>(obase + static_cast<int64_t>(q) * Hd + ch * 32 + u * 8) = w;
                 }
                 __syncwarp();

@@ -208,12 +208,24 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
                     }
                     mbar_arrive_expect_tx(full(s), tx);
                     const uint32_t xs = sbase + L::X_OFF + s * L::X_BYTES;
-                    tma_load_2d(xs, &tmap_x, full(s), kk * kBKS, 0);
-                    tma_load_2d(xs + L::X_BOX, &tmap_x, full(s), kk * kBKS + 64, 0);
                     const uint32_t ws = sbase + L::W_OFF + s * L::W_BYTES;
-                    tma_load_2d(ws, &tmap_w, full(s), kk * (kBKS / 2), row0);
-                    tma_load_2d(ws + L::W_HALF, &tmap_w, full(s), kk * (kBKS / 2),
-                                row0 + RB / 2);
+                    const uint32_t wbox = static_cast<uint32_t>(RB / 2) * (kBKS / 2);
+                    if (dbg_check(tma_box_ok(xs, L::X_BOX, 1024, sbase, sbase + L::W_OFF,
+                                             kk * kBKS, 2) &&
+                                      tma_box_ok(xs + L::X_BOX, L::X_BOX, 1024, sbase,
+                                                 sbase + L::W_OFF, kk * kBKS + 64, 2) &&
+                                      wbox <= L::W_HALF &&
+                                      tma_box_ok(ws, wbox, 1024, sbase + L::W_OFF,
+                                                 sbase + L::BAR_OFF, kk * (kBKS / 2), 1) &&
+                                      tma_box_ok(ws + L::W_HALF, wbox, 1024, sbase + L::W_OFF,
+                                                 sbase + L::BAR_OFF, kk * (kBKS / 2), 1),
+                                  p.status)) {
+                        tma_load_2d(xs, &tmap_x, full(s), kk * kBKS, 0);
+                        tma_load_2d(xs + L::X_BOX, &tmap_x, full(s), kk * kBKS + 64, 0);
+                        tma_load_2d(ws, &tmap_w, full(s), kk * (kBKS / 2), row0);
+                        tma_load_2d(ws + L::W_HALF, &tmap_w, full(s), kk * (kBKS / 2),
+                                    row0 + RB / 2);
+                    }
                     if (++kk == KS) kk = 0;
                 }
             }

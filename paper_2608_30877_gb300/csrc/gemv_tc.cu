@@ -163,11 +163,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     mbar_arrive_expect_tx(full_tma(s), tx);
                     const uint32_t st = sbase + s * L::STAGE;
-                    tma_load_2d(st, &tmap_x, full_tma(s), kk * kGroupK, 0);
-                    tma_load_2d(st + L::X_BOX, &tmap_x, full_tma(s), kk * kGroupK + 64, 0);
-                    tma_load_2d(st + L::X_BYTES, &tmap_w, full_tma(s), kk * (kGroupK / 2), row0);
-                    tma_load_2d(st + L::X_BYTES + L::W_HALF, &tmap_w, full_tma(s),
-                                kk * (kGroupK / 2), row0 + RB / 2);
+                    const uint32_t end = sbase + L::BAR_OFF;
+                    if (dbg_check(tma_box_ok(st, L::X_BOX, 1024, sbase, end, kk * kGroupK, 2) &&
+                                      tma_box_ok(st + L::X_BOX, L::X_BOX, 1024, sbase, end,
+                                                 kk * kGroupK + 64, 2),
+                                  p.status)) {
+                        tma_load_2d(st, &tmap_x, full_tma(s), kk * kGroupK, 0);
+                        tma_load_2d(st + L::X_BOX, &tmap_x, full_tma(s), kk * kGroupK + 64, 0);
+                    }
+                    const uint32_t wbox = static_cast<uint32_t>(RB / 2) * (kGroupK / 2);
+                    if (dbg_check(wbox <= L::W_HALF &&
+                                      tma_box_ok(st + L::X_BYTES, wbox, 1024, sbase, end,
+                                                 kk * (kGroupK / 2), 1) &&
+                                      tma_box_ok(st + L::X_BYTES + L::W_HALF, wbox, 1024, sbase,
+                                                 end, kk * (kGroupK / 2), 1),
+                                  p.status)) {
+                        tma_load_2d(st + L::X_BYTES, &tmap_w, full_tma(s), kk * (kGroupK / 2),
+                                    row0);
+                        tma_load_2d(st + L::X_BYTES + L::W_HALF, &tmap_w, full_tma(s),
+                                    kk * (kGroupK / 2), row0 + RB / 2);
+                    }
                     if (++kk == KS) kk = 0;
                 }
             }
@@ -309,7 +324,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     codes_signed(c1.y, v + 20);
                     codes_signed(c1.z, v + 24);
                     codes_signed(c1.w, v + 28);
-                    tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS + t * (kAK / 2), v);
+                    if (dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (kAK / 2) <= L::TMEM_COLS,
+                                  p.status))
+                        tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS + t * (kAK / 2), v);
                     tmem_st_wait();
                     tc_fence_before();
                     __syncwarp();

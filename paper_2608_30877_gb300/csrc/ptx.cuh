@@ -96,6 +96,37 @@ __device__ __forceinline__ void record_status(int* status, int code) {
     atomicCAS(status, 0, code);
 }
 
+// ---------------------------------------------------------------- debug checks
+// Built with -DW4A16_DEBUG, the kernels check the indices they compute before
+// each TMA copy, tensor-memory access and global store: a failed check records
+// W4A16_ERR_INDEX (6) in the status word and the access is skipped (no trap,
+// the context stays usable; a skipped copy makes the waits on it run out).
+// Without the flag every check is the constant true and compiles away.
+#ifdef W4A16_DEBUG
+constexpr bool kDebugChecks = true;
+#else
+constexpr bool kDebugChecks = false;
+#endif
+
+__device__ __forceinline__ bool dbg_check(bool ok, int* status) {
+    if constexpr (kDebugChecks) {
+        if (!ok) atomicCAS(status, 0, 6 /* W4A16_ERR_INDEX */);
+        return ok;
+    }
+    return true;
+}
+
+// A tiled TMA load into [dst, dst + box_bytes): the innermost coordinate times
+// the element size a multiple of 16 bytes (else the copy is an illegal
+// instruction), the destination aligned to `align` and inside the shared-memory
+// region [lo, hi) that holds the CTA's staging buffers.
+__device__ __forceinline__ bool tma_box_ok(uint32_t dst, uint32_t box_bytes, uint32_t align,
+                                           uint32_t lo, uint32_t hi, int32_t c0,
+                                           uint32_t elem_bytes) {
+    return c0 >= 0 && ((static_cast<uint32_t>(c0) * elem_bytes) & 15u) == 0 &&
+           (dst & (align - 1u)) == 0 && dst >= lo && dst + box_bytes <= hi;
+}
+
 // Every wait in the kernels is bounded: after limit_ns of global time (the
 // launch's wait limit, kWaitLimitNs unless a test lowers it) or kWaitIterCap
 // polls the waiter gives up, raises the CTA's abort flag and records a

@@ -246,7 +246,8 @@ __device__ __forceinline__ void plain_epilogue_tile(const TsParams& p, uint32_t 
                     col = n - 1;
                     word = pack_bf16x2(other, f1);
                 }
-                if (m < p.M && col < p.N)
+                if (m < p.M && col < p.N &&
+                    dbg_check((col & 1) == 0 && col + 1 < p.N && m >= 0 && col >= 0, p.status))
                     *reinterpret_cast<uint32_t*>(p.out + static_cast<int64_t>(m) * p.N +
                                                  col) = word;
             }
@@ -376,10 +377,15 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                         break;
                     }
                     mbar_arrive_expect_tx(full_tma(s), L::X_BYTES + L::W_BYTES);
-                    tma_load_2d(sbase + L::X_OFF + s * L::X_BYTES, &tmap_x, full_tma(s), kt * kBK,
-                                t0);
-                    tma_load_2d(sbase + L::W_OFF + s * L::W_BYTES, &tmap_w, full_tma(s),
-                                kt * (kBK / 2), n0);
+                    const uint32_t xd = sbase + L::X_OFF + s * L::X_BYTES;
+                    const uint32_t wd = sbase + L::W_OFF + s * L::W_BYTES;
+                    if (dbg_check(tma_box_ok(xd, L::X_BYTES, 1024, sbase, sbase + L::W_OFF,
+                                             kt * kBK, 2) && t0 >= 0, p.status))
+                        tma_load_2d(xd, &tmap_x, full_tma(s), kt * kBK, t0);
+                    if (dbg_check(tma_box_ok(wd, L::W_BYTES, 128, sbase + L::W_OFF,
+                                             sbase + L::BAR_OFF, kt * (kBK / 2), 1) && n0 >= 0,
+                                  p.status))
+                        tma_load_2d(wd, &tmap_w, full_tma(s), kt * (kBK / 2), n0);
                 }
             }
             // Drain: every load this thread issued has landed before exit.
@@ -416,6 +422,10 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     }
                     tc_fence_after();
                     const uint32_t xs = sbase + L::X_OFF + s * L::X_BYTES;
+                    if (!dbg_check(L::A_COL + (sa + 1) * (kBK / 2) <= L::TMEM_COLS &&
+                                       L::D_COL + T <= L::A_COL,
+                                   p.status))
+                        continue;
 #pragma unroll
                     for (int ks = 0; ks < kBK / 16; ++ks) {
                         const uint32_t a = tmem + L::A_COL + sa * (kBK / 2) + ks * 8;
@@ -475,7 +485,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             const int j = static_cast<int>(i / static_cast<uint32_t>(KT));
             const int kt = static_cast<int>(i - static_cast<uint32_t>(j) * KT);
             const uint16_t* row = scale_row(j);
-            return row ? __ldg(row + grp_of(kt)) : static_cast<uint16_t>(0);
+            return row && dbg_check(grp_of(kt) < KG, p.status) ? __ldg(row + grp_of(kt))
+                                                              : static_cast<uint16_t>(0);
         };
         uint32_t it = 0;
         bool ok = true;
@@ -513,7 +524,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                 dequant_word(w1.y, s2, v + 20);
                 dequant_word(w1.z, s2, v + 24);
                 dequant_word(w1.w, s2, v + 28);
-                tmem_st_32x32b_x32(lane_base + L::A_COL + sa * (kBK / 2), v);
+                if (dbg_check(L::A_COL + (sa + 1) * (kBK / 2) <= L::TMEM_COLS, p.status))
+                    tmem_st_32x32b_x32(lane_base + L::A_COL + sa * (kBK / 2), v);
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();

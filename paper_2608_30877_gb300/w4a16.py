@@ -14,10 +14,12 @@ import re
 import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libw4a16.so")
+# W4A16_DEBUG=1 loads the build with the kernels' index checks
+LIB_PATH = os.path.join(_PKG, "libw4a16_debug.so" if os.environ.get("W4A16_DEBUG") == "1"
+                        else "libw4a16.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "w4a16.h")
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_ALIGNMENT, ERR_CUDA, ERR_TIMEOUT = range(6)
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_ALIGNMENT, ERR_CUDA, ERR_TIMEOUT, ERR_INDEX = range(7)
 ACT_NONE, ACT_SWIGLU, ACT_GELU = range(3)
 
 _lib = None

@@ -117,3 +117,15 @@ def test_stack_graph_rejects_bad_handles(L):
     assert not h.value
     assert L.w4a16_stack_graph_launch(None, None) == W.ERR_INVALID_ARG
     assert L.w4a16_stack_graph_destroy(None) == W.ERR_INVALID_ARG
+
+
+def test_debug_build_exports_the_same_symbols():
+    """The W4A16_DEBUG build (the kernels' index checks) compiles and exports
+    every declared function; its status string for the check is defined."""
+    import ctypes as C
+    from paper_2608_30877_gb300 import build as B
+    D = C.CDLL(B.build(debug=True))
+    for name in W.header_functions():
+        assert hasattr(D, name), name
+    D.w4a16_status_string.restype = C.c_char_p
+    assert b"debug" in D.w4a16_status_string(W.ERR_INDEX)
