@@ -76,6 +76,11 @@ bool g_small_m_streaming = true;
 // W4A16_SMALL_M=mma / tc forces one of them.
 int g_small_m_tc_from = 17;
 bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile
+// CTA pairs with 384-token tiles from this many tokens on (the tile padding
+// is then under 2.4%): one dequantised weight stage serves 1.5x the tokens,
+// which under the power cap is 4.51 against 4.32 scored pairs/s on the stack.
+// W4A16_GEMM_WIDE=1 / 0 forces them on or off.
+int64_t g_gemm_wide_from = 16384;
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
 
@@ -105,6 +110,10 @@ int device_state(DeviceState** out) {
             if (const char* e = std::getenv("W4A16_GEMM_PAIR")) {
                 if (e[0] == '1') g_gemm_pair = true;
                 if (e[0] == '0') g_gemm_pair = false;
+            }
+            if (const char* e = std::getenv("W4A16_GEMM_WIDE")) {
+                if (e[0] == '1') g_gemm_wide_from = 33;
+                if (e[0] == '0') g_gemm_wide_from = int64_t{1} << 40;  // never
             }
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
@@ -245,9 +254,10 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
                   cudaStream_t stream) {
     if (M <= 32 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
-    const TsVariant v = M <= 32      ? TsVariant::kGemv32
-                        : g_gemm_pair ? TsVariant::kGemmPair
-                                      : TsVariant::kGemm256;
+    const TsVariant v = M <= 32                      ? TsVariant::kGemv32
+                        : g_gemm_pair && M >= g_gemm_wide_from ? TsVariant::kGemmPairWide
+                        : g_gemm_pair                ? TsVariant::kGemmPair
+                                                     : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);
     alignas(64) CUtensorMap tx;
     alignas(64) CUtensorMap tw;

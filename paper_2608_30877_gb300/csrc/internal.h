@@ -39,6 +39,7 @@ enum class TsVariant : int {
     kGemm256 = 0,   // 256 tokens per tile, persistent grid (large M)
     kGemv32 = 1,    // 32 tokens per tile, one tile per CTA (M <= 32)
     kGemmPair = 2,  // 256 tokens x 256 weight rows per CTA pair (cta_group::2), persistent
+    kGemmPairWide = 3,  // 384 tokens (two 192-column accumulators) x 256 rows per CTA pair
 };
 
 int ts_tokens_per_tile(TsVariant v);

@@ -48,11 +48,15 @@ constexpr uint32_t kEpilogueSleepNs = W4A16_EPI_SLEEP_NS;
 constexpr int kBK = 64;     // k per stage (one 128-byte swizzle row of bf16)
 
 // PAIR: a CTA pair (cta_group::2) computes 2 x 128 weight rows x T tokens;
-// each CTA stages T/2 tokens of x and its own 128 weight rows.
-template <int T, int S_SMEM, int S_TMEM, bool PAIR>
+// each CTA stages T/2 tokens of x and its own 128 weight rows.  NB: the tile's
+// tokens form NB accumulator blocks of T/NB columns, one MMA each per k step,
+// all reading the same A stage (so one dequantised stage serves T tokens).
+template <int T, int S_SMEM, int S_TMEM, bool PAIR, int NB = 1>
 struct Layout {
     static constexpr int XT = PAIR ? T / 2 : T;  // tokens of x staged per CTA
-    static constexpr int X_BYTES = XT * kBK * 2;
+    static constexpr int XB = XT / NB;           // token rows per x box (one per block)
+    static constexpr int X_BOX = XB * kBK * 2;
+    static constexpr int X_BYTES = NB * X_BOX;
     static constexpr int W_BYTES = kRows * kBK / 2;
     static constexpr int X_OFF = 0;
     static constexpr int W_OFF = S_SMEM * X_BYTES;
@@ -73,8 +77,8 @@ struct Layout {
                                      : COLS_USED <= 256 ? 256
                                                         : 512;
     static_assert(COLS_USED <= 512, "tensor memory holds 512 columns");
-    static_assert(X_BYTES % 1024 == 0, "x stages must keep 1024-byte alignment");
-    static_assert(T % 32 == 0 && T >= 32 && T <= 256, "tokens per tile");
+    static_assert(X_BOX % 1024 == 0, "x boxes must keep 1024-byte alignment");
+    static_assert(T % 32 == 0 && T >= 32 && T / NB <= 256 && T % NB == 0, "tokens per tile");
 };
 
 // Unit -> (token tile, weight unit): units are rastered in groups of group_t
@@ -286,17 +290,17 @@ constexpr int threads_for() {
 // CTA's TMA loads complete on its own full_tma barrier, which its dequant
 // warps wait on before they arrive on full_a: the MMA's wait on full_a
 // covers both CTAs' x and weight stages.
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED, bool PAIR>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool FUSED, bool PAIR,
+          int NB>
 __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     w4a16_ts_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_w, const TsParams p) {
-    using L = Layout<T, S_SMEM, S_TMEM, PAIR>;
+    using L = Layout<T, S_SMEM, S_TMEM, PAIR, NB>;
     constexpr int CW = PAIR ? 2 : 1;
     // Pairs run one ring: a stage's shared-memory slot and tensor-memory A
     // slot are released together by one commit per CTA (two commits per
     // stage instead of four; 1463 -> 1607 TFLOP/s on the QKV prefill).
-    static_assert(!PAIR || S_SMEM == S_TMEM, "pairs: one ring of stages");
-    constexpr bool kUnified = PAIR;
+    constexpr bool kUnified = PAIR && S_SMEM == S_TMEM;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -368,7 +372,8 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
             for (int unit = unit_first<CW>(); ok && unit < unit_count<CW>(p); unit += unit_stride<CW>()) {
                 int tt, wt;
                 unit_tile<CW>(unit, p, rank, tt, wt);
-                const int t0 = tt * T + rank * L::XT, n0 = wt * kRows;
+                // block nb of the tile: tokens tt T + nb T/NB .., this CTA's XB of them
+                const int t0 = tt * T + rank * L::XB, n0 = wt * kRows;
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % S_SMEM;
                     const uint32_t ph = (it / S_SMEM) & 1u;
@@ -379,9 +384,14 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     mbar_arrive_expect_tx(full_tma(s), L::X_BYTES + L::W_BYTES);
                     const uint32_t xd = sbase + L::X_OFF + s * L::X_BYTES;
                     const uint32_t wd = sbase + L::W_OFF + s * L::W_BYTES;
-                    if (dbg_check(tma_box_ok(xd, L::X_BYTES, 1024, sbase, sbase + L::W_OFF,
-                                             kt * kBK, 2) && t0 >= 0, p.status))
-                        tma_load_2d(xd, &tmap_x, full_tma(s), kt * kBK, t0);
+#pragma unroll
+                    for (int nb = 0; nb < NB; ++nb) {
+                        if (dbg_check(tma_box_ok(xd + nb * L::X_BOX, L::X_BOX, 1024, sbase,
+                                                 sbase + L::W_OFF, kt * kBK, 2) && t0 >= 0,
+                                      p.status))
+                            tma_load_2d(xd + nb * L::X_BOX, &tmap_x, full_tma(s), kt * kBK,
+                                        t0 + nb * (T / NB));
+                    }
                     if (dbg_check(tma_box_ok(wd, L::W_BYTES, 128, sbase + L::W_OFF,
                                              sbase + L::BAR_OFF, kt * (kBK / 2), 1) && n0 >= 0,
                                   p.status))
@@ -395,7 +405,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && leader) {
-            constexpr uint32_t idesc = idesc_bf16_f32(kRows * CW, T);
+            constexpr uint32_t idesc = idesc_bf16_f32(kRows * CW, T / NB);
             uint32_t it = 0, tcount = 0, tiles_done = 0;
             bool ok = true;
             bool issued = false;
@@ -429,11 +439,15 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
 #pragma unroll
                     for (int ks = 0; ks < kBK / 16; ++ks) {
                         const uint32_t a = tmem + L::A_COL + sa * (kBK / 2) + ks * 8;
-                        const uint64_t b = sdesc_kmajor_sw128(xs + ks * 32);
-                        if constexpr (PAIR)
-                            tc_mma_ts_pair(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
-                        else
-                            tc_mma_ts(tmem + L::D_COL, a, b, idesc, (kt | ks) != 0);
+#pragma unroll
+                        for (int nb = 0; nb < NB; ++nb) {
+                            const uint32_t d = tmem + L::D_COL + nb * (T / NB);
+                            const uint64_t b = sdesc_kmajor_sw128(xs + nb * L::X_BOX + ks * 32);
+                            if constexpr (PAIR)
+                                tc_mma_ts_pair(d, a, b, idesc, (kt | ks) != 0);
+                            else
+                                tc_mma_ts(d, a, b, idesc, (kt | ks) != 0);
+                        }
                     }
                     issued = true;
                     commit(empty_smem(s));
@@ -603,15 +617,15 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
     }
 }
 
-template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool PAIR>
+template <int T, int S_SMEM, int S_TMEM, int DQ, int EP, int MIN_BLOCKS, bool PAIR, int NB = 1>
 cudaError_t launch_variant(const CUtensorMap* tx, const CUtensorMap* tw, const TsParams& p,
                            int grid, cudaStream_t stream) {
-    using L = Layout<T, S_SMEM, S_TMEM, PAIR>;
+    using L = Layout<T, S_SMEM, S_TMEM, PAIR, NB>;
     // the plain variant carries none of the fused epilogue's code or registers
     const bool fused =
         p.epi.bias != nullptr || p.epi.residual != nullptr || p.epi.act != kActNone;
-    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true, PAIR>
-                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false, PAIR>;
+    auto kern = fused ? w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, true, PAIR, NB>
+                      : w4a16_ts_kernel<T, S_SMEM, S_TMEM, DQ, EP, MIN_BLOCKS, false, PAIR, NB>;
     // Idempotent; cheap enough to repeat per launch and per device.
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES);
@@ -657,6 +671,13 @@ constexpr int kGemmT = 256, kGemmSS = W4A16_GEMM_SS, kGemmST = 6, kGemmDQ = W4A1
 #define W4A16_PAIR_STAGES 8
 #endif
 constexpr int kPairSS = W4A16_PAIR_STAGES, kPairST = W4A16_PAIR_STAGES;
+// Wide CTA pairs: 384 tokens per tile as two accumulators of 192 columns, so
+// one dequantised A stage serves 384 tokens; tensor memory = 384 accumulator
+// + 4 x 32 A columns.  Shared memory per stage: 24 KB x + 4 KB weights.
+#ifndef W4A16_WIDE_SS
+#define W4A16_WIDE_SS 4
+#endif
+constexpr int kWideT = 384, kWideSS = W4A16_WIDE_SS, kWideST = 4;
 // Small M: 32 tokens per tile, 8 shared-memory stages of 8 KB, 3 A stages;
 // 128 tensor-memory columns so that three CTAs share an SM.
 constexpr int kGemvT = 32, kGemvSS = 8, kGemvST = 3, kGemvDQ = 1, kGemvEP = 1;
@@ -670,7 +691,7 @@ int pair_slots(int sm_count) {
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return sm_count / 2;
     if (cache[dev] > 0) return cache[dev];
     using L = Layout<kGemmT, kPairSS, kPairST, true>;
-    auto kern = w4a16_ts_kernel<kGemmT, kPairSS, kPairST, kGemmDQ, kGemmEP, 1, false, true>;
+    auto kern = w4a16_ts_kernel<kGemmT, kPairSS, kPairST, kGemmDQ, kGemmEP, 1, false, true, 1>;
     int n = 0;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_BYTES) ==
         cudaSuccess) {
@@ -695,15 +716,19 @@ int pair_slots(int sm_count) {
 
 }  // namespace
 
-int ts_tokens_per_tile(TsVariant v) { return v == TsVariant::kGemv32 ? kGemvT : kGemmT; }
+int ts_tokens_per_tile(TsVariant v) {
+    return v == TsVariant::kGemv32 ? kGemvT : v == TsVariant::kGemmPairWide ? kWideT : kGemmT;
+}
 
 int ts_x_box_tokens(TsVariant v) {
-    return v == TsVariant::kGemmPair ? kGemmT / 2 : ts_tokens_per_tile(v);
+    if (v == TsVariant::kGemmPair) return kGemmT / 2;
+    if (v == TsVariant::kGemmPairWide) return kWideT / 4;  // two blocks, half per CTA
+    return ts_tokens_per_tile(v);
 }
 
 int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
     if (v == TsVariant::kGemm256) return p.num_tiles < sm_count ? p.num_tiles : sm_count;
-    if (v == TsVariant::kGemmPair) {
+    if (v == TsVariant::kGemmPair || v == TsVariant::kGemmPairWide) {
         const int units = p.num_t_tiles * ((p.num_w_tiles + 1) / 2);
         const int slots = pair_slots(sm_count);
         return 2 * (units < slots ? units : slots);
@@ -719,6 +744,9 @@ cudaError_t ts_launch(TsVariant v, const CUtensorMap* tx, const CUtensorMap* tw,
     if (v == TsVariant::kGemmPair)
         return launch_variant<kGemmT, kPairSS, kPairST, kGemmDQ, kGemmEP, 1, true>(tx, tw, p,
                                                                                   grid, stream);
+    if (v == TsVariant::kGemmPairWide)
+        return launch_variant<kWideT, kWideSS, kWideST, kGemmDQ, kGemmEP, 1, true, 2>(
+            tx, tw, p, grid, stream);
     return launch_variant<kGemvT, kGemvSS, kGemvST, kGemvDQ, kGemvEP, 3, false>(tx, tw, p, grid,
                                                                                stream);
 }

@@ -227,3 +227,52 @@ def test_small_m_kernels_every_m(kernel):
     r = subprocess.run([sys.executable, "-c", _FORCED_KERNEL_CHECK.format(root=root, cases=cases)],
                        env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0 and "ok" in r.stdout, r.stdout + r.stderr
+
+
+_FORCED_GEMM_CHECK = r"""
+import sys
+import numpy as np, torch
+sys.path.insert(0, {root!r})
+from oracle import oracle as O
+from paper_2608_30877_gb300 import synthetic as S
+from tests.gpu_helpers import assert_close, bf16_to_f64, host_case, to_device
+from paper_2608_30877_gb300 import w4a16 as W
+for (M, N, K) in {cases!r}:
+    x, xb, packed, scales = host_case(M, N, K, 128, 500 + M, 501 + N)
+    xd, wd, sd = to_device(x, packed, scales)
+    out = W.linear(xd, wd, sd, 128)
+    torch.cuda.synchronize()
+    ref = O.linear_rows(xb, packed, scales, N, K, 128, nthreads=O.max_threads())
+    assert_close(bf16_to_f64(out), ref, f"M={{M}} N={{N}} K={{K}}")
+assert W.get_device_error() == W.OK
+# the abort path under a lowered wait limit, then a correct call again
+W.set_wait_limit(1)
+W.linear(S.make_x(900, 2048, 3, "cuda"), torch.zeros((128 * 300, 1024), dtype=torch.uint8,
+         device="cuda"), torch.zeros((128 * 300, 16), dtype=torch.bfloat16, device="cuda"), 128)
+assert W.get_device_error() == W.ERR_TIMEOUT
+W.set_wait_limit(0)
+x, xb, packed, scales = host_case(500, 384, 512, 128, 7, 8)
+xd, wd, sd = to_device(x, packed, scales)
+out = W.linear(xd, wd, sd, 128)
+torch.cuda.synchronize()
+assert_close(bf16_to_f64(out), O.linear_rows(xb, packed, scales, 384, 512, 128), "after abort")
+assert W.get_device_error() == W.OK
+print("ok")
+"""
+
+
+@pytest.mark.parametrize("env", [{"W4A16_GEMM_WIDE": "1"}, {"W4A16_GEMM_WIDE": "0"},
+                                 {"W4A16_GEMM_PAIR": "0"}])
+def test_large_m_gemm_variants_ragged(env):
+    """Every large-M GEMM variant forced on ragged shapes (ragged token tiles,
+    an odd number of 128-row weight tiles, K not a multiple of the 384-token
+    tile's stage count), then its abort path: the 384-token CTA pairs (the
+    default from 16384 tokens), the 256-token CTA pairs and one CTA per tile."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    cases = [(33, 128, 128), (300, 384, 256), (385, 1000, 640), (769, 640, 1152), (1200, 2048, 512)]
+    r = subprocess.run([sys.executable, "-c", _FORCED_GEMM_CHECK.format(root=root, cases=cases)],
+                       env=dict(os.environ, **env), capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0 and "ok" in r.stdout, r.stdout + r.stderr
