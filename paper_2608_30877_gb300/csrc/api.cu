@@ -68,7 +68,12 @@ struct DeviceState {
 std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
-int g_group_t = 6;  // raster group, token tiles (stack sweep: 2-16, best 3 and 6)
+// Raster groups, in token tiles: 6 of 256 tokens (stack sweep 2-16: best 3
+// and 6), 3 of 384 (stack at 1 / 2 / 3 / 4 / 6 / 8: 4.49 / 4.59 / 4.60-4.66 /
+// 4.59 / 4.52 / 4.50 pairs/s).  W4A16_GROUP_T sets both.
+int g_group_t = 6;
+int g_group_t_wide = 3;
+int64_t g_group_bytes = 0;  // if > 0: groups sized so that a group's x takes at most this
 bool g_small_m_streaming = true;
 // Small M on the tcgen05 streaming kernel above this many tokens, on the
 // warp-level mma.sync kernel up to it (12288 x 49152: M = 32 108 against
@@ -115,9 +120,13 @@ int device_state(DeviceState** out) {
                 if (e[0] == '1') g_gemm_wide_from = 33;
                 if (e[0] == '0') g_gemm_wide_from = int64_t{1} << 40;  // never
             }
+            if (const char* e = std::getenv("W4A16_GROUP_BYTES")) {
+                const long long v = std::atoll(e);
+                if (v > 0) g_group_bytes = v;
+            }
             if (const char* e = std::getenv("W4A16_GROUP_T")) {
                 const int v = std::atoi(e);
-                if (v > 0 && v <= 4096) g_group_t = v;
+                if (v > 0 && v <= 4096) g_group_t = g_group_t_wide = v;
             }
         }
         if (cudaDeviceGetAttribute(&st.sm_count, cudaDevAttrMultiProcessorCount, dev) !=
@@ -278,7 +287,12 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     p.num_t_tiles = static_cast<int>((M + T - 1) / T);
     p.num_w_tiles = static_cast<int>((N + 127) / 128);
     p.num_tiles = p.num_t_tiles * p.num_w_tiles;
-    p.group_t = v == TsVariant::kGemv32 ? 1 : g_group_t;
+    p.group_t = v == TsVariant::kGemv32 ? 1 : v == TsVariant::kGemmPairWide ? g_group_t_wide : g_group_t;
+    if (v != TsVariant::kGemv32 && g_group_bytes > 0) {
+        const int64_t per_tile = static_cast<int64_t>(T) * K * 2;
+        const int64_t gt = g_group_bytes / per_tile;
+        p.group_t = static_cast<int>(gt < 1 ? 1 : gt > 64 ? 64 : gt);
+    }
     p.epi = epi;
     p.wait_ns = wait_limit_ns();
     const int grid = ts_grid(v, p, st.sm_count);
