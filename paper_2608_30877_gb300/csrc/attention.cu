@@ -43,7 +43,8 @@ namespace {
 constexpr int kD = 128;        // head dimension
 constexpr int kBQ = 128;       // queries per job (MMA M)
 constexpr int kBKV = 64;       // keys per block (MMA N of S, K of PV)
-constexpr int kThreads = 6 * 32;  // TMA warp, MMA warp, 4 softmax warps
+constexpr int kPvWarp = 6;
+constexpr int kThreads = 7 * 32;  // TMA warp, S-MMA warp, 4 softmax warps, PV-MMA warp
 
 struct AttnLayout {
     static constexpr int QBOX = kBQ * 128;    // one [128 rows x 64 cols] bf16 box: 16 KB
@@ -58,8 +59,8 @@ struct AttnLayout {
     static constexpr int STAGE_WARP = 32 * 64;
     static constexpr int BAR_OFF = STAGE_OFF + 4 * STAGE_WARP;
     // q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2],
-    // s_full[2], p_full[2], o_ready[2], drain
-    static constexpr int NBARS = 17;
+    // s_full[2], p_full[2], o_ready[2], drain[2]
+    static constexpr int NBARS = 18;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 32 + 1024;
     // tensor memory columns: two S buffers (blocks alternate; P of a block is
@@ -281,7 +282,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     // PV products only now and then (hence two o_ready).
     auto p_full = [&](uint32_t b) { return bars + 96u + 8u * b; };
     auto o_ready = [&](uint32_t b) { return bars + 112u + 8u * b; };
-    const uint32_t drain = bars + 128u;
+    auto drain = [&](uint32_t i) { return bars + 128u + 8u * i; };
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
     int* bad_flag = reinterpret_cast<int*>(smem + L::MISC_OFF + 8);
@@ -308,7 +309,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 mbar_init(p_full(i), 4);  // one arrival per softmax warp
                 mbar_init(o_ready(i), 1);
             }
-            mbar_init(drain, 1);
+            mbar_init(drain(0), 1);
+            mbar_init(drain(1), 1);
             *abort_flag = 0;
             fence_mbar_init();
             prefetch_tmap(&tmap_q);
@@ -404,43 +406,63 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (uint32_t i = nv > 2 ? nv - 2 : 0; i < nv; ++i) settle(v_full(i & 1u), (i >> 1) & 1u);
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        // S runs two blocks ahead of PV: S of block g + 2 goes into S buffer
-        // g & 1 as soon as the PV product of block g has read P from it, so it
-        // overlaps the softmax of block g + 1.
+        // ------------------------------------------------------------ MMA issuers
+        // Two threads: this warp's issues the S products, warp 6's the PV
+        // products, each waiting only on what its own products need and
+        // committing its own barriers, so neither's waits hold up the other's
+        // MMAs.  S runs two blocks ahead of PV: S of block g + 2 goes into S
+        // buffer g & 1 as soon as the PV product of block g has read P from
+        // it, so it overlaps the softmax of block g + 1.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBQ, kBKV);
-        constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
         bool ok = run;
-        auto issue_s = [&](const BlockWalk& w, uint32_t gs) -> bool {
-            const uint32_t b = gs & 1u;
-            if (w.j == 0 && !wait_one(q_full, w.jn & 1u, abort_flag, p.status, p.wait_ns)) return false;
-            if (!wait_one(k_full(b), (gs >> 1) & 1u, abort_flag, p.status, p.wait_ns)) return false;
-            tc_fence_after();
-            const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + b * L::KV_TILE;
-#pragma unroll
-            for (int kk = 0; kk < kD / 16; ++kk) {
-                tc_mma_ss(tmem + L::S_COL + b * kBKV,
-                          sdesc_kmajor_sw128(qs + (kk >> 2) * L::QBOX + (kk & 3) * 32),
-                          sdesc_kmajor_sw128(ks + (kk >> 2) * L::KBOX + (kk & 3) * 32), idesc_s,
-                          kk > 0 ? 1u : 0u);
-            }
-            tc_commit(s_full(b));
-            tc_commit(k_empty(b));
-            if (w.j == w.nblk - 1) tc_commit(q_empty);  // the job's last S product frees Q
-            return true;
-        };
-        BlockWalk ws, wp;  // the next block to take its S product, the next for its PV product
+        BlockWalk ws;  // the next block to take its S product
         if (ok) {
             ws.t = t_first;
             walk_job(p, njobs, lane, ws);
-            wp = ws;
         }
-        uint32_t gs = 0, g = 0;
-        for (int k = 0; k < 2 && ok && ws.valid; ++k, ++gs) {
-            if (lane == 0) ok = issue_s(ws, gs);
+        uint32_t gs = 0;
+        while (ok && ws.valid) {
+            const uint32_t b = gs & 1u;
+            if (lane == 0) {
+                // the buffer's previous block (gs - 2) has had its PV product
+                ok = gs < 2 || wait_one(o_ready(b), ((gs - 2) >> 1) & 1u, abort_flag, p.status,
+                                        p.wait_ns);
+                if (ok && ws.j == 0)
+                    ok = wait_one(q_full, ws.jn & 1u, abort_flag, p.status, p.wait_ns);
+                if (ok) ok = wait_one(k_full(b), (gs >> 1) & 1u, abort_flag, p.status, p.wait_ns);
+                if (ok) {
+                    tc_fence_after();
+                    const uint32_t qs = sbase + L::Q_OFF, ks = sbase + L::K_OFF + b * L::KV_TILE;
+#pragma unroll
+                    for (int kk = 0; kk < kD / 16; ++kk) {
+                        tc_mma_ss(tmem + L::S_COL + b * kBKV,
+                                  sdesc_kmajor_sw128(qs + (kk >> 2) * L::QBOX + (kk & 3) * 32),
+                                  sdesc_kmajor_sw128(ks + (kk >> 2) * L::KBOX + (kk & 3) * 32),
+                                  idesc_s, kk > 0 ? 1u : 0u);
+                    }
+                    tc_commit(s_full(b));
+                    tc_commit(k_empty(b));
+                    if (ws.j == ws.nblk - 1) tc_commit(q_empty);  // the job's last S frees Q
+                }
+            }
             ok = __shfl_sync(0xffffffffu, ok, 0);
+            ++gs;
             walk_next(p, njobs, t_step, lane, ws);
         }
+        if (lane == 0) {
+            tc_commit(drain(0));  // every MMA issued has completed before tensor memory is freed
+            settle(drain(0), 0);
+        }
+    } else if (warp == kPvWarp) {
+        // ------------------------------------------------------------ PV issuer
+        constexpr uint32_t idesc_o = idesc_bf16_f32(kBQ, kD) | (1u << 16);  // B MN-major
+        bool ok = run;
+        BlockWalk wp;  // the next block to take its PV product
+        if (ok) {
+            wp.t = t_first;
+            walk_job(p, njobs, lane, wp);
+        }
+        uint32_t g = 0;
         while (ok && wp.valid) {
             const uint32_t b = g & 1u;
             if (lane == 0) {
@@ -461,20 +483,14 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tc_commit(o_ready(b));
                     tc_commit(v_empty(b));
                 }
-                if (ok && ws.valid)
-                    ok = wait_one(o_ready(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns) && issue_s(ws, gs);
             }
             ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (ws.valid) {
-                ++gs;
-                walk_next(p, njobs, t_step, lane, ws);
-            }
             ++g;
             walk_next(p, njobs, t_step, lane, wp);
         }
         if (lane == 0) {
-            tc_commit(drain);  // every MMA issued has completed before tensor memory is freed
-            settle(drain, 0);
+            tc_commit(drain(1));
+            settle(drain(1), 0);
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue
