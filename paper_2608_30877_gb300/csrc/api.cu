@@ -274,7 +274,7 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
                        ts_x_box_tokens(v), CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != W4A16_OK) return rc;
     rc = encode_2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, w, K / 2, N, K / 2, 32, 128,
-                   CU_TENSOR_MAP_SWIZZLE_NONE);
+                   CU_TENSOR_MAP_SWIZZLE_32B);
     if (rc != W4A16_OK) return rc;
     TsParams p;
     p.scales = static_cast<const uint16_t*>(s);

@@ -392,7 +392,7 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                             tma_load_2d(xd + nb * L::X_BOX, &tmap_x, full_tma(s), kt * kBK,
                                         t0 + nb * (T / NB));
                     }
-                    if (dbg_check(tma_box_ok(wd, L::W_BYTES, 128, sbase + L::W_OFF,
+                    if (dbg_check(tma_box_ok(wd, L::W_BYTES, 256, sbase + L::W_OFF,
                                              sbase + L::BAR_OFF, kt * (kBK / 2), 1) && n0 >= 0,
                                   p.status))
                         tma_load_2d(wd, &tmap_w, full_tma(s), kt * (kBK / 2), n0);
@@ -524,10 +524,13 @@ __global__ void __launch_bounds__(threads_for<DQ, EP>(), MIN_BLOCKS)
                     break;
                 }
                 tc_fence_after();
-                const uint4* wrow =
-                    reinterpret_cast<const uint4*>(smem + L::W_OFF + s * L::W_BYTES + r * 32);
-                const uint4 w0 = wrow[0];
-                const uint4 w1 = wrow[1];
+                // the weight box comes with the 32-byte swizzle: the two 16-byte
+                // halves of rows 4-7 of every 8 are swapped, so the 8 lanes of a
+                // load phase read 8 distinct bank groups
+                const uint8_t* wrow = smem + L::W_OFF + s * L::W_BYTES + r * 32;
+                const uint32_t swz = static_cast<uint32_t>((r >> 2) & 1) * 16u;
+                const uint4 w0 = *reinterpret_cast<const uint4*>(wrow + swz);
+                const uint4 w1 = *reinterpret_cast<const uint4*>(wrow + (16u ^ swz));
                 const uint32_t s2 = splat_bf16(s_cur);
                 uint32_t v[32];
                 dequant_word(w0.x, s2, v + 0);
