@@ -3,8 +3,8 @@
 //
 // Design, GB300-first:
 //   - persistent grid, one CTA per SM; CTA c owns a contiguous range of RB
-//     weight rows (RB a multiple of 16, at most 352), so every SM streams the
-//     same number of bytes -- no tile-count quantisation;
+//     weight rows (RB even, at most 352), so every SM streams the same number
+//     of bytes -- no tile-count quantisation;
 //   - one shared-memory stage covers 128 k = one scale group (g = 128): two
 //     TMA boxes of RB/2 rows x 64 B of packed weights (64-byte swizzle) and
 //     two 128-byte-swizzled boxes of x (T = 8, 16 or 32 token rows; rows >= M
@@ -508,8 +508,11 @@ cudaError_t launch_gemv_variant(const CUtensorMap* tx, const CUtensorMap* tw,
 }  // namespace
 
 int gemv_rows_per_cta(int64_t N, int sm_count) {
+    // even (SwiGLU pairs rows 2j, 2j+1 within a CTA); the compute warps mask
+    // the rows of their last tile past RB, so RB need not fill whole tiles and
+    // every SM gets a range (12288 x 49152: 324 rows on 152 SMs, not 336 on 147)
     int64_t per = (N + sm_count - 1) / sm_count;
-    per = (per + 15) / 16 * 16;
+    per = (per + 1) / 2 * 2;
     if (per > kRowsMax) per = kRowsMax;
     if (per < 16) per = 16;
     return static_cast<int>(per);

@@ -56,7 +56,7 @@ struct GemvParams {
     uint16_t* out;           // bf16 bits [M, N]
     int* status;
     int M, N, K, g;
-    int rows_per_cta;        // RB: weight rows per CTA chunk, multiple of 16, <= 384
+    int rows_per_cta;        // RB: weight rows per CTA chunk, even, <= 352 (<= 384 tcgen05)
     int num_chunks;          // ceil(N / RB)
     int nt;                  // MMA tiles per chunk: ceil(RB / 128)
     Epilogue epi;
