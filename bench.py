@@ -38,20 +38,24 @@ METRIC = "W4A16 GEMM TFLOP/s & % of roofline; scored pairs/s on 175B-class linea
 # workload and by a hash of the kernel's sources at capture time: once the
 # kernel changes the hash no longer matches and traffic is reported as null.
 NCU_TRAFFIC = {
-    # mean of one launch per stack shape at M = 8192, scaled by 8 to M = 65536
-    # (profiles/gemm_pair_stack_traffic_m8192.md)
-    ("stack", "ts", "0e169a7ecb79efe6"): 3.67e9 * 8,
-    # QKV prefill 4096x12288x36864, one launch (full capture)
-    ("qkv", "ts", "0e169a7ecb79efe6"): 1.280e9 + 0.292e9,
-    # small-M readout, M = 8, 12288x49152 (DRAM counters of one launch)
-    ("gemv", "gemv", "aacb64e0363a16ed"): 0.31868e9 + 0.00322e9,
+    # mean of one launch per stack shape at M = 16384 (384-token tiles, as in
+    # the benched stack), scaled by 4 to M = 65536
+    # (profiles/gemm_pair_wide_stack_traffic_m16384.md)
+    ("stack", "ts", "99063559ec7b3d82"): 7.1207e9 * 4,
+    # QKV prefill 4096x12288x36864 (256-token CTA pairs), one launch (full capture)
+    ("qkv", "ts", "99063559ec7b3d82"): 1.2102e9 + 0.2921e9,
+    # small-M readout, M = 8 (warp-level kernel), 12288x49152, one launch
+    ("gemv", "gemv", "270f49f687deb1b3"): 0.31859e9 + 0.00380e9,
+    # small-M readout, M = 32 (tensor-core kernel), 12288x49152, one launch
+    ("gemv32", "gemvtc", "684b8b4e8d570de2"): 0.32650e9 + 0.00355e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
     # one 8-pair launch); scaled by pairs / 8 for the benched launch
-    ("attention", "attn", "04bc02017fef4c26"): 0.8508e9 + 0.1827e9,
+    ("attention", "attn", "3294a8d7153edae5"): 0.8125e9 + 0.1834e9,
 }
 
 KERNEL_FILES = {"ts": ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"),
                 "gemv": ("gemv_rows.cu", "dequant.cuh", "ptx.cuh"),
+                "gemvtc": ("gemv_tc.cu", "dequant.cuh", "ptx.cuh"),
                 "attn": ("attention.cu",)}
 
 
@@ -71,6 +75,8 @@ def ncu_traffic(config: str, m: int, pairs: int = 8):
         t = NCU_TRAFFIC.get((config, "attn", kernel_source_hash("attn")))
         return None if t is None else t * pairs / 8  # qkv and out grow with the pairs
     if config == "gemv":
+        if 17 <= m <= 32:  # the tensor-core kernel; the capture is of M = 32
+            return NCU_TRAFFIC.get(("gemv32", "gemvtc", kernel_source_hash("gemvtc")))
         if m > 8:  # the capture is of the M <= 8 instantiation
             return None
         kind = "gemv"
