@@ -758,10 +758,12 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
         ach, peak, unit = wl.bytes / t / 1e9, peaks["hbm_gbs"], "GB/s"
     else:
         ach, peak, unit = wl.flops / t / 1e12, peaks["bf16_tflops"], "TFLOP/s"
+    traffic = (ncu_traffic("qkv", lc.M) if name == "qkv_prefill"
+               else ncu_traffic("gemv", lc.M) if hbm else None)
     res = {"workload": lc.name, "value": ach, "unit": unit, "us_per_launch": t * 1e6,
            "launches": steps, "clocks": clk.summary(),
            "roofline": {"bound": "hbm" if hbm else "tensor", "achieved": ach, "peak": peak,
-                        "unit": unit, "frac": ach / peak,
+                        "unit": unit, "frac": ach / peak, "traffic": traffic,
                         "peak_source": peaks["source"] + (" hbm_gbs" if hbm else " bf16_tflops"),
                         "algorithmic_bytes": wl.bytes, "flops": wl.flops},
            "l2": ("weights rotate over 2 copies larger than L2" if copies > 1
