@@ -85,6 +85,12 @@ def ncu_traffic(config: str, m: int, pairs: int = 8):
     return NCU_TRAFFIC.get((config, kind, kernel_source_hash(kind)))
 
 
+# The GB300's nominal dense bf16 tensor rate and HBM3e bandwidth: each
+# roofline also carries its fraction of these (frac_nominal).
+NOMINAL_BF16_TFLOPS = 2250.0
+NOMINAL_HBM_GBS = 8000.0
+
+
 def load_peaks() -> dict:
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -665,7 +671,9 @@ def main():
         peak = peaks["bf16_tflops_sustained"] if args.config == "stack" else peaks["bf16_tflops"]
         roof = {"bound": "tensor", "unit": "TFLOP/s"}
     traffic = ncu_traffic(args.config, args.m, args.pairs)
+    nominal = NOMINAL_HBM_GBS if roof["bound"] == "hbm" else NOMINAL_BF16_TFLOPS
     roof.update({"achieved": achieved, "peak": peak, "frac": achieved / peak,
+                 "frac_nominal": achieved / nominal,
                  "traffic": traffic, "peak_source": peaks["source"] + (
                      " bf16_tflops_sustained" if args.config == "stack" else
                      (" hbm_gbs" if args.config in ("gemv", "topk") else " bf16_tflops")),
@@ -744,13 +752,21 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
             wl.step()
         b.record(stream)
         b.synchronize()
-        steps = max(10, int(seconds / (a.elapsed_time(b) / 2e3)))
-        a.record(stream)
-        for _ in range(steps):
-            wl.step()
-        b.record(stream)
-        b.synchronize()
-    t = a.elapsed_time(b) / 1e3 / steps
+        # the timed region as 10 back-to-back repetitions, each bracketed by
+        # its own events: the mean over all launches and the spread of the
+        # per-launch time over the repetitions
+        reps = 10
+        per_rep = max(1, int(seconds / (a.elapsed_time(b) / 2e3)) // reps)
+        steps = reps * per_rep
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(reps + 1)]
+        ev[0].record(stream)
+        for r in range(reps):
+            for _ in range(per_rep):
+                wl.step()
+            ev[r + 1].record(stream)
+        ev[-1].synchronize()
+    rep_us = sorted(ev[r].elapsed_time(ev[r + 1]) * 1e3 / per_rep for r in range(reps))
+    t = ev[0].elapsed_time(ev[-1]) / 1e3 / steps
     if W.get_device_error() != W.OK:
         raise RuntimeError(f"device status word set during {name}")
     hbm = lc.M <= 32
@@ -761,9 +777,15 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
     traffic = (ncu_traffic("qkv", lc.M) if name == "qkv_prefill"
                else ncu_traffic("gemv", lc.M) if hbm else None)
     res = {"workload": lc.name, "value": ach, "unit": unit, "us_per_launch": t * 1e6,
-           "launches": steps, "clocks": clk.summary(),
+           "launches": steps,
+           "us_per_launch_reps": {"reps": reps, "launches_per_rep": per_rep,
+                                  "median": (rep_us[reps // 2 - 1] + rep_us[reps // 2]) / 2,
+                                  "min": rep_us[0], "max": rep_us[-1]},
+           "clocks": clk.summary(),
            "roofline": {"bound": "hbm" if hbm else "tensor", "achieved": ach, "peak": peak,
-                        "unit": unit, "frac": ach / peak, "traffic": traffic,
+                        "unit": unit, "frac": ach / peak,
+                        "frac_nominal": ach / (NOMINAL_HBM_GBS if hbm else NOMINAL_BF16_TFLOPS),
+                        "traffic": traffic,
                         "peak_source": peaks["source"] + (" hbm_gbs" if hbm else " bf16_tflops"),
                         "algorithmic_bytes": wl.bytes, "flops": wl.flops},
            "l2": ("weights rotate over 2 copies larger than L2" if copies > 1
