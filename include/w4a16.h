@@ -79,16 +79,17 @@ typedef enum {
  *   scales_bf16  [N, K/g] bf16, device
  *   out_bf16     [M, N]   bf16, device, written in full
  * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 32 with
- * g = 128 runs the bandwidth-bound row-range streaming kernel; other small
- * M (g != 128) run the tcgen05 kernel with 32-token tiles.  The tcgen05
- * kernels multiply x by the dequantised weights wd defined above, so they
- * differ from each other only in the fp32 summation order.  The streaming
- * kernel factors the scale out of each group instead: it sums x * (code - 8)
- * over the group exactly in fp32 (the codes are small integers) and adds
- * scale * that sum, so it never rounds (code - 8) * scale to bf16.  Both
- * stay within the same error bound of the exact product x * wd^T (fp32
- * accumulation followed by one bf16 rounding of the output); they are not
- * bit-identical to each other.
+ * g = 128 runs a bandwidth-bound row-range streaming kernel (warp-level
+ * MMAs for M <= 16, tcgen05 for M = 17..32); other small M (g != 128) run
+ * the tcgen05 GEMM with 32-token tiles.  The tcgen05 kernels multiply x by
+ * the dequantised weights wd defined above, so they differ from each other
+ * only in the fp32 summation order.  The warp-level streaming kernel factors
+ * the scale out of each group instead: it sums x * (code - 8) over the group
+ * exactly in fp32 (the codes are small integers) and adds scale * that sum,
+ * so it never rounds (code - 8) * scale to bf16.  Both stay within the same
+ * error bound of the exact product x * wd^T (fp32 accumulation followed by
+ * one bf16 rounding of the output); they are not bit-identical to each
+ * other.
  */
 int w4a16_linear(const void* x_bf16, const void* w_packed_u8, const void* scales_bf16,
                  void* out_bf16, int64_t M, int64_t N, int64_t K, int64_t g,

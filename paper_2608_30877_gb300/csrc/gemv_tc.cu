@@ -2,16 +2,20 @@
 // tensor core: the bandwidth-bound regime where the whole packed weight
 // matrix streams from HBM once per call.
 //
-// out[m, n] = sum_groups s[n, grp] * (sum_{k in grp} x[m, k] * (q[n, k] - 8)).
+// out[m, n] = sum_k x[m, k] * wd[n, k],   wd = RNE_bf16((q[n, k] - 8) * s[n, k / g])
+//
+// (the same weights as w4a16_dequant and the large-M GEMM: the result differs
+// from theirs only in the fp32 summation order).
 //
 // Why the tensor core here: at M = 16-32 tokens the matmul is 19-39 GFLOP per
 // call, and warp-level mma.sync runs at ~610 TFLOP/s on this GPU -- 32-64 us,
-// more than the ~46 us the weights take to stream.  tcgen05.mma has four
-// times that rate and runs asynchronously, leaving the SM's integer pipes to
-// the unpacking.
+// more than the ~46 us the weights take to stream.  tcgen05.mma runs
+// asynchronously, leaving the SM's integer and half-precision pipes to the
+// dequantisation.
 //
 // Per CTA (persistent, one per SM): a contiguous range of RB <= 384 weight
-// rows (RB = N / #SMs rounded up to even), as three MMA tiles of 128 rows.
+// rows (RB = N / #SMs rounded up to even), as three MMA tiles of 128 rows,
+// each with ONE fp32 accumulator in tensor memory for the whole K walk.
 // Per scale group of 128 k:
 //   warp 0      TMA: two 64-k boxes of x (NTOK token rows, 128-byte swizzle,
 //               rows >= M zero-filled) and two boxes of RB/2 rows x 64 B of
@@ -19,20 +23,20 @@
 //   warp 2      reorders each staged x chunk in place into the (k, k+4) pair
 //               order in which the codes come out of a packed word;
 //   warps 4-15  dequant: thread = one weight row of one tile (its TMEM lane);
-//               per 64 k, 8 words -> the exact bf16 pairs q - 8 (shift,
-//               three-input LOP3, one bf16x2 subtraction per pair; no scale
-//               multiply) -> tcgen05.st into a ring of SA A stages;
-//   warps 1, 3  one thread each, taking the groups in turn, issues
-//               D_grp[128 x NTOK] = A[128 x 16] x B[NTOK x 16]^T for the three
-//               tiles (A from tensor memory, B = x in shared memory), 24 MMAs
-//               per group, into its own accumulator buffer: the group's sum
-//               of x (q - 8), exact products accumulated in fp32;
-//   warps 16-27 fold: tcgen05.ld of the group's accumulator, acc += s * D in
-//               fp32 registers (thread = row, NTOK accumulators), then the
-//               (fused) epilogue from registers.
-// The scale is applied once per group and row in fp32 (as in the warp-level
-// streaming kernel), so (q - 8) * s is never rounded to bf16; the result stays
-// within the same error bound of x * wd^T.
+//               per 64 k, 8 words -> bf16 pairs (q - 8) * s (shift,
+//               three-input LOP3, one bf16x2 subtraction and one bf16x2
+//               multiply per pair) -> tcgen05.st into a ring of SA A stages;
+//               after the last group, the epilogue: tcgen05.ld of the row's
+//               NTOK accumulators, then the (fused) epilogue from registers;
+//   warps 1, 3, 16  one thread each, one per tile, issues
+//               D_t[128 x NTOK] += A_t[128 x 16] x B[NTOK x 16]^T (A from
+//               tensor memory, B = x in shared memory), 8 MMAs per group,
+//               accumulating into its tile's accumulator.
+// With the scale applied in the dequant there is no per-group accumulator to
+// fold: nothing waits on the MMAs inside the K walk except the A ring.  A
+// single thread issues these small MMAs at ~130 SM clocks each, slower than
+// the tensor pipe runs them, hence one issuing thread (and one A ring and
+// accumulator hand-off) per tile.
 //
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
 // W4A16_ERR_TIMEOUT, drains its copies and MMAs, frees tensor memory and
@@ -50,34 +54,42 @@ constexpr int kTiles = 3;                 // MMA tiles of 128 rows per CTA
 constexpr int kRowsMax = 128 * kTiles;    // rows per CTA chunk
 constexpr int kGroupK = 128;              // k per TMA stage = one scale group
 constexpr int kAK = 64;                   // k per tensor-memory A stage
-constexpr int kFirstDequantWarp = 4;      // warps 4..15 (warp % 4 = TMEM sub-partition)
-constexpr int kFirstFoldWarp = 16;        // warps 16..27
-constexpr int kRowWarps = 4 * kTiles;     // dequant (and fold) warps
-constexpr int kThreads = 32 * (kFirstFoldWarp + kRowWarps);
+constexpr int kFirstRowWarp = 4;          // warps 4..15 (warp % 4 = TMEM sub-partition)
+constexpr int kRowWarps = 4 * kTiles;     // dequant + epilogue warps
+constexpr int kLastIssuerWarp = kFirstRowWarp + kRowWarps;  // warp 16: tile 2's MMAs
+constexpr int kThreads = 32 * (kLastIssuerWarp + 1);
+
+// MMA-issuing warp of tile t: 1, 3, 16.
+__device__ __forceinline__ int issuer_tile(int warp) {
+    return warp == 1 ? 0 : warp == 3 ? 1 : warp == kLastIssuerWarp ? 2 : -1;
+}
 
 template <int NTOK>
 struct TLayout {
     static_assert(NTOK == 16 || NTOK == 32, "MMA N for M = 128");
     static constexpr int S = NTOK == 32 ? 6 : 7;                     // TMA stage slots
-    static constexpr int SA = NTOK == 32 ? 3 : 4;                    // A stage slots
+    static constexpr int SA = 4;                                     // A stage slots
     static constexpr int X_BOX = NTOK * 128;                         // 64 k x NTOK tokens
     static constexpr int X_BYTES = 2 * X_BOX;
     static constexpr int W_HALF = (kRowsMax / 2) * (kGroupK / 2);    // 192 rows x 64 B
     static constexpr int W_BYTES = 2 * W_HALF;
     static constexpr int STAGE = X_BYTES + W_BYTES;                  // x, then the weights
-    // full_tma[S], empty_smem[S], x_ready[S], full_a[SA], empty_a[SA],
-    // d_full[2], d_empty[2], drain[2]
+    // full_tma[S], empty_smem[S], x_ready[S], then per tile: full_a[SA],
+    // empty_a[SA], d_full, d_empty, drain
     static constexpr int BAR_OFF = S * STAGE;
-    static constexpr int NBARS = 3 * S + 2 * SA + 6;
+    static constexpr int TILE_BARS = 2 * SA + 3;
+    static constexpr int NBARS = 3 * S + kTiles * TILE_BARS;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;          // + 1024-B alignment slack
-    // tensor memory: two accumulator buffers (kTiles x NTOK columns each),
-    // then SA A stages (kTiles x 32 columns each: 64 k of bf16 pairs)
+    // tensor memory: the accumulators (kTiles x NTOK columns) at column 0,
+    // then from column 128 SA A stages (kTiles x 32 columns each: 64 k of
+    // bf16 pairs)
     static constexpr int D_COLS = kTiles * NTOK;
-    static constexpr int A_COL = 2 * D_COLS;
+    static constexpr int A_COL = 128;
     static constexpr int A_COLS = kTiles * (kAK / 2);
     static constexpr int TMEM_COLS = 512;
-    static_assert(A_COL + SA * A_COLS <= TMEM_COLS, "tensor memory holds 512 columns");
+    static_assert(D_COLS <= A_COL && A_COL + SA * A_COLS <= TMEM_COLS,
+                  "tensor memory holds 512 columns");
     static_assert(X_BOX % 1024 == 0 && W_HALF % 1024 == 0 && STAGE % 1024 == 0,
                   "swizzled boxes keep 1024-byte alignment");
     static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
@@ -102,30 +114,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto full_tma = [&](int s) { return bars + 8u * s; };
     auto empty_smem = [&](int s) { return bars + 8u * (S + s); };
     auto x_ready = [&](int s) { return bars + 8u * (2 * S + s); };
-    auto full_a = [&](int a) { return bars + 8u * (3 * S + a); };
-    auto empty_a = [&](int a) { return bars + 8u * (3 * S + SA + a); };
-    auto d_full = [&](int b) { return bars + 8u * (3 * S + 2 * SA + b); };
-    auto d_empty = [&](int b) { return bars + 8u * (3 * S + 2 * SA + 2 + b); };
-    auto drain = [&](int i) { return bars + 8u * (3 * S + 2 * SA + 4 + i); };
+    auto tile_bar = [&](int t, int i) { return bars + 8u * (3 * S + t * L::TILE_BARS + i); };
+    auto full_a = [&](int t, int a) { return tile_bar(t, a); };
+    auto empty_a = [&](int t, int a) { return tile_bar(t, SA + a); };
+    auto d_full = [&](int t) { return tile_bar(t, 2 * SA); };
+    auto d_empty = [&](int t) { return tile_bar(t, 2 * SA + 1); };
+    auto drain = [&](int t) { return tile_bar(t, 2 * SA + 2); };
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::MISC_OFF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::MISC_OFF + 4);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_tma(s), 1);
-            mbar_init(empty_smem(s), kRowWarps + 1);  // every dequant warp read W, the MMAs read x
+            // every row warp of the p.nt tiles in use has read W, and every
+            // such tile's MMAs have read x
+            mbar_init(empty_smem(s), 5 * p.nt);
             mbar_init(x_ready(s), 1);
         }
-        for (int a = 0; a < SA; ++a) {
-            mbar_init(full_a(a), kRowWarps);
-            mbar_init(empty_a(a), 1);
+        for (int t = 0; t < kTiles; ++t) {
+            for (int a = 0; a < SA; ++a) {
+                mbar_init(full_a(t, a), 4);  // the tile's four row warps
+                mbar_init(empty_a(t, a), 1);
+            }
+            mbar_init(d_full(t), 1);
+            mbar_init(d_empty(t), 4);
+            mbar_init(drain(t), 1);
         }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(d_full(b), 1);
-            mbar_init(d_empty(b), kRowWarps);
-        }
-        mbar_init(drain(0), 1);
-        mbar_init(drain(1), 1);
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tmap_x);
@@ -190,67 +204,60 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t last = it < static_cast<uint32_t>(S) ? it : S;
             for (uint32_t i = it - last; i < it; ++i) settle(full_tma(i % S), (i / S) & 1u);
         }
-    } else if (warp == 1 || warp == 3) {
+    } else if (issuer_tile(warp) >= 0) {
         // ------------------------------------------------------------ MMA issuers
-        // Two threads take the groups in turn (warp 1 the even ones, with
-        // accumulator buffer 0; warp 3 the odd ones, buffer 1): one thread's
-        // commits and waits overlap the other's MMAs, and each commit tracks
-        // only its own thread's MMAs.
-        if (lane == 0) {
-            const uint32_t mine = warp == 1 ? 0u : 1u;
+        // (tiles past the chunk's rows, t >= p.nt, are not computed)
+        const int t = issuer_tile(warp);
+        if (lane == 0 && t < p.nt) {
             constexpr uint32_t idesc = idesc_bf16_f32(128, NTOK);
-            uint32_t it = 0, ia = 0;
+            uint32_t it = 0, ia = 0, nchunk = 0;
             bool ok = true, issued = false;
-            for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
+            for (int chunk = blockIdx.x; ok && chunk < p.num_chunks;
+                 chunk += gridDim.x, ++nchunk) {
+                // the epilogue has read the previous chunk's accumulators
+                if (nchunk > 0 &&
+                    !wait_one(d_empty(t), (nchunk - 1u) & 1u, abort_flag, p.status, p.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
                 for (int g = 0; ok && g < KS; ++g, ++it) {
-                    if ((it & 1u) != mine) {
-                        ia += kGroupK / kAK;
-                        continue;
-                    }
                     const int s = it % S;
-                    const int b = it & 1;  // accumulator buffer of this group
-                    if (!wait_one(x_ready(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns) ||
-                        !wait_one(d_empty(b), ((it >> 1) & 1u) ^ 1u, abort_flag, p.status,
-                                  p.wait_ns)) {
+                    if (!wait_one(x_ready(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    // descriptors and addresses of the group: one add per MMA
                     const uint64_t bdesc = sdesc_kmajor_sw128(sbase + s * L::STAGE);
-                    const uint32_t dcol = tmem + b * L::D_COLS;
                     for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
                         const int a = ia % SA;
-                        if (!wait_one(full_a(a), (ia / SA) & 1u, abort_flag, p.status, p.wait_ns)) {
+                        if (!wait_one(full_a(t, a), (ia / SA) & 1u, abort_flag, p.status,
+                                      p.wait_ns)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        // consecutive MMAs go to the three tiles' accumulators in
-                        // turn, so that none waits for the one before it
 #pragma unroll
                         for (int ks = 0; ks < kAK / 16; ++ks) {
-#pragma unroll
-                            for (int t = 0; t < kTiles; ++t) {
-                                // the descriptor's start address is in 16-byte units
-                                tc_mma_ts(dcol + t * NTOK,
-                                          tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
-                                          bdesc + static_cast<uint64_t>((h * L::X_BOX + ks * 32) >> 4),
-                                          idesc, (h | ks) != 0);
-                            }
+                            // the descriptor's start address is in 16-byte units
+                            tc_mma_ts(tmem + t * NTOK,
+                                      tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
+                                      bdesc + static_cast<uint64_t>((h * L::X_BOX + ks * 32) >> 4),
+                                      idesc, (g | h | ks) != 0);
                         }
                         issued = true;
-                        tc_commit(empty_a(a));
+                        tc_commit(empty_a(t, a));
                     }
                     if (!ok) break;
-                    tc_commit(d_full(b));
                     tc_commit(empty_smem(s));
                 }
+                if (!ok) break;
+                tc_commit(d_full(t));  // the chunk's accumulators of tile t are final
             }
             if (issued) {
                 // every MMA issued has completed before tensor memory is freed
-                tc_commit(drain(mine));
-                settle(drain(mine), 0);
+                tc_commit(drain(t));
+                settle(drain(t), 0);
             }
         }
     } else if (warp == 2) {
@@ -278,11 +285,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(x_ready(s));
             }
         }
-    } else if (warp >= kFirstDequantWarp && warp < kFirstFoldWarp) {
-        // ------------------------------------------------------------ dequant
-        const int t = (warp - kFirstDequantWarp) >> 2;  // MMA tile
-        const int sub = warp & 3;                       // TMEM sub-partition
-        const int r = t * 128 + sub * 32 + lane;        // local row
+    } else if (warp >= kFirstRowWarp && warp < kLastIssuerWarp &&
+               (warp - kFirstRowWarp) / 4 < p.nt) {
+        // ------------------------------------------------------------ dequant + epilogue
+        const int t = (warp - kFirstRowWarp) >> 2;  // MMA tile
+        const int sub = warp & 3;                   // TMEM sub-partition
+        const int r = t * 128 + sub * 32 + lane;    // local row
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
         // the row's four 16-byte chunks in a stage (64-byte swizzle)
         const bool in_range = r < RB;
@@ -290,12 +298,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int rr = in_range ? r - bx * (RB / 2) : 0;
         const uint32_t row_off = L::X_BYTES + bx * L::W_HALF + rr * (kGroupK / 2);
         const uint32_t swz = static_cast<uint32_t>((rr >> 1) & 3);
-        uint32_t it = 0, ia = 0;
+        uint32_t it = 0, ia = 0, nchunk = 0;
         bool ok = true;
-        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
-            const bool valid = in_range && chunk * RB + r < p.N;
+        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x, ++nchunk) {
+            const int n = chunk * RB + r;
+            const bool valid = in_range && n < p.N;
+            // the row's scales in the rotated group order, one group ahead
+            const uint16_t* srow = p.scales + static_cast<int64_t>(valid ? n : 0) * KS;
+            int kk = rot;
+            uint16_t s_next = __ldg(srow + kk);
             for (int g = 0; ok && g < KS; ++g, ++it) {
                 const int s = it % S;
+                const uint32_t s2 = valid ? splat_bf16(s_next) : 0u;
+                if (++kk == KS) kk = 0;
+                if (g + 1 < KS) s_next = __ldg(srow + kk);
                 if (!wait_warp(full_tma(s), (it / S) & 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
@@ -309,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         c0 = lds128(wrow + 16u * ((2u * h) ^ swz));
                         c1 = lds128(wrow + 16u * ((2u * h + 1u) ^ swz));
                     }
-                    if (!wait_warp(empty_a(a), ((ia / SA) & 1u) ^ 1u, abort_flag, p.status,
+                    if (!wait_warp(empty_a(t, a), ((ia / SA) & 1u) ^ 1u, abort_flag, p.status,
                                    p.wait_ns)) {
                         ok = false;
                         break;
@@ -324,61 +340,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                     codes_signed(c1.y, v + 20);
                     codes_signed(c1.z, v + 24);
                     codes_signed(c1.w, v + 28);
+                    // wd = RNE_bf16((q - 8) * s): the exact q - 8 times the scale, one rounding
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = bf16x2_mul(v[j], s2);
                     if (dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (kAK / 2) <= L::TMEM_COLS,
                                   p.status))
                         tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS + t * (kAK / 2), v);
                     tmem_st_wait();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(full_a(a));
+                    if (lane == 0) mbar_arrive(full_a(t, a));
                 }
                 if (!ok) break;
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty_smem(s));  // this warp's weight reads are done
             }
-        }
-    } else if (warp >= kFirstFoldWarp) {
-        // ------------------------------------------------------------ fold + epilogue
-        const int t = (warp - kFirstFoldWarp) >> 2;
-        const int sub = warp & 3;
-        const int r = t * 128 + sub * 32 + lane;
-        const uint32_t d_base = tmem + (static_cast<uint32_t>(sub * 32) << 16) + t * NTOK;
-        uint32_t it = 0;
-        bool ok = true;
-        for (int chunk = blockIdx.x; ok && chunk < p.num_chunks; chunk += gridDim.x) {
-            const int n = chunk * RB + r;
-            const bool valid = r < RB && n < p.N;
-            const uint16_t* srow = p.scales + static_cast<int64_t>(valid ? n : 0) * KS;
+            if (!ok) break;
+            // ---- epilogue: the row's NTOK accumulators, tokens 0 .. M - 1
+            if (!wait_warp(d_full(t), nchunk & 1u, abort_flag, p.status, p.wait_ns)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
             float acc[NTOK];
 #pragma unroll
-            for (int j = 0; j < NTOK; ++j) acc[j] = 0.0f;
-            int kk = rot;
-            uint16_t s_next = __ldg(srow + kk);
-            for (int g = 0; g < KS; ++g, ++it) {
-                const int b = it & 1;
-                const float sc = valid ? bf16_to_f32(s_next) : 0.0f;
-                if (++kk == KS) kk = 0;
-                if (g + 1 < KS) s_next = __ldg(srow + kk);
-                if (!wait_warp(d_full(b), (it >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
+            for (int half = 0; half < NTOK / 16; ++half) {
+                uint32_t d[16];
+                tmem_ld_32x32b_x16(lane_base + t * NTOK + half * 16, d);
+                tmem_ld_wait_x16(d);
 #pragma unroll
-                for (int half = 0; half < NTOK / 16; ++half) {
-                    uint32_t v[16];
-                    tmem_ld_32x32b_x16(d_base + b * L::D_COLS + half * 16, v);
-                    tmem_ld_wait_x16(v);
-#pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        acc[half * 16 + j] = fmaf(sc, __uint_as_float(v[j]), acc[half * 16 + j]);
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(d_empty(b));
+                for (int j = 0; j < 16; ++j) acc[half * 16 + j] = __uint_as_float(d[j]);
             }
-            if (!ok) break;
-            // ---- epilogue from registers: row n, tokens 0 .. M - 1
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(d_empty(t));  // the next chunk's MMAs may overwrite D
             const Epilogue& ep = p.epi;
             if constexpr (!FUSED) {
 #pragma unroll
