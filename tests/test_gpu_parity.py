@@ -229,6 +229,24 @@ def test_small_m_kernels_every_m(kernel):
     assert r.returncode == 0 and "ok" in r.stdout, r.stdout + r.stderr
 
 
+@pytest.mark.parametrize("kernel", ["tc", "mma"])
+def test_small_m_kernels_several_chunks_per_cta(kernel):
+    """More weight rows than one row range per SM can hold (RB is capped at
+    384 rows for the tensor-core kernel, 352 for the warp-level one), so some
+    CTAs walk a second chunk: the tensor-core kernel's accumulator hand-off
+    between chunks and both kernels' stage rings across chunks, on every
+    output against the oracle."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    cases = [(M, 60010, 256) for M in (3, 16, 24, 32)]
+    env = dict(os.environ, W4A16_SMALL_M=kernel)
+    r = subprocess.run([sys.executable, "-c", _FORCED_KERNEL_CHECK.format(root=root, cases=cases)],
+                       env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0 and "ok" in r.stdout, r.stdout + r.stderr
+
+
 _FORCED_GEMM_CHECK = r"""
 import sys
 import numpy as np, torch
