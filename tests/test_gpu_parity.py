@@ -184,6 +184,7 @@ def test_error_codes_launch_nothing():
     (1, 1, 128, 128), (3, 100, 256, 128), (8, 1000, 1024, 128), (16, 4096, 512, 128),
     (17, 1234, 384, 128), (32, 8192, 256, 64), (32, 50000, 128, 128), (9, 77, 2048, 256),
     (8, 60000, 640, 128), (24, 60000, 1152, 128), (2, 53600, 2176, 128),
+    (20, 1, 128, 128), (29, 130, 128, 128),
 ])
 def test_small_m_streaming_kernel_shapes(M, N, K, g):
     """M <= 32 with g = 128 runs the row-range streaming kernel: ragged row
