@@ -50,7 +50,7 @@ int ts_grid(TsVariant v, const TsParams& p, int sm_count);
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                       const TsParams& p, int grid, cudaStream_t stream);
 
-// Parameters of the small-M streaming kernel (gemv_rows.cu).
+// Parameters of the small-M streaming kernels (gemv_rows.cu, gemv_tc.cu).
 struct GemvParams {
     const uint16_t* scales;  // bf16 bits [N, K/g]
     uint16_t* out;           // bf16 bits [M, N]
@@ -58,7 +58,7 @@ struct GemvParams {
     int M, N, K, g;
     int rows_per_cta;        // RB: weight rows per CTA chunk, even, <= 352 (<= 384 tcgen05)
     int num_chunks;          // ceil(N / RB)
-    int nt;                  // MMA tiles per chunk: ceil(RB / 128)
+    int nt;                  // tcgen05 kernel: 128-row MMA tiles per chunk, ceil(RB / 128)
     Epilogue epi;
     uint64_t wait_ns;
 };
