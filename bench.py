@@ -47,7 +47,7 @@ NCU_TRAFFIC = {
     # small-M readout, M = 8 (warp-level kernel), 12288x49152, one launch
     ("gemv", "gemv", "270f49f687deb1b3"): 0.31859e9 + 0.00380e9,
     # small-M readout, M = 32 (tensor-core kernel), 12288x49152, one launch
-    ("gemv32", "gemvtc", "63fd2f374e9e3cf7"): 0.32640e9 + 0.00366e9,
+    ("gemv32", "gemvtc", "88cfd3cc92630dc4"): 0.32655e9 + 0.00339e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
     # one 8-pair launch); scaled by pairs / 8 for the benched launch
     ("attention", "attn", "3294a8d7153edae5"): 0.8125e9 + 0.1834e9,

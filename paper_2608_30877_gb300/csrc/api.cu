@@ -76,8 +76,8 @@ int g_group_t_wide = 3;
 int64_t g_group_bytes = 0;  // if > 0: groups sized so that a group's x takes at most this
 bool g_small_m_streaming = true;
 // Small M on the tcgen05 streaming kernel from this many tokens on, on the
-// warp-level mma.sync kernel below it (12288 x 49152: M = 32 97 against
-// 128 us; M = 16 99 against 83 us; M = 8 99 against 68 us).
+// warp-level mma.sync kernel below it (12288 x 49152: M = 32 94 against
+// 128 us; M = 16 95 against 83 us; M = 8 95 against 68 us).
 // W4A16_SMALL_M=mma / tc forces one of them.
 int g_small_m_tc_from = 17;
 bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile

@@ -23,9 +23,10 @@
 //   warp 2      reorders each staged x chunk in place into the (k, k+4) pair
 //               order in which the codes come out of a packed word;
 //   warps 4-15  dequant: thread = one weight row of one tile (its TMEM lane);
-//               per 64 k, 8 words -> bf16 pairs (q - 8) * s (shift,
+//               per scale group, 16 words -> bf16 pairs (q - 8) * s (shift,
 //               three-input LOP3, one bf16x2 subtraction and one bf16x2
-//               multiply per pair) -> tcgen05.st into a ring of SA A stages;
+//               multiply per pair) -> tcgen05.st into a ring of SA A stages
+//               (one per group);
 //               after the last group, the epilogue: tcgen05.ld of the row's
 //               NTOK accumulators, then the (fused) epilogue from registers;
 //   warps 1, 3, 16  one thread each, one per tile, issues
@@ -53,7 +54,12 @@ namespace {
 constexpr int kTiles = 3;                 // MMA tiles of 128 rows per CTA
 constexpr int kRowsMax = 128 * kTiles;    // rows per CTA chunk
 constexpr int kGroupK = 128;              // k per TMA stage = one scale group
-constexpr int kAK = 64;                   // k per tensor-memory A stage
+#ifndef W4A16_TC_AK
+#define W4A16_TC_AK 128
+#endif
+constexpr int kAK = W4A16_TC_AK;          // k per tensor-memory A stage (64 or 128)
+static_assert(kAK == 64 || kAK == 128, "A stages of half or whole scale groups");
+constexpr int kChunks = kAK / 32;         // 16-byte chunks (32 codes) per row and A stage
 constexpr int kFirstRowWarp = 4;          // warps 4..15 (warp % 4 = TMEM sub-partition)
 constexpr int kRowWarps = 4 * kTiles;     // dequant + epilogue warps
 constexpr int kLastIssuerWarp = kFirstRowWarp + kRowWarps;  // warp 16: tile 2's MMAs
@@ -68,7 +74,8 @@ template <int NTOK>
 struct TLayout {
     static_assert(NTOK == 16 || NTOK == 32, "MMA N for M = 128");
     static constexpr int S = NTOK == 32 ? 6 : 7;                     // TMA stage slots
-    static constexpr int SA = 4;                                     // A stage slots
+    // A stage slots: as many as fit next to the accumulators
+    static constexpr int SA = kAK == 64 ? 4 : 2;
     static constexpr int X_BOX = NTOK * 128;                         // 64 k x NTOK tokens
     static constexpr int X_BYTES = 2 * X_BOX;
     static constexpr int W_HALF = (kRowsMax / 2) * (kGroupK / 2);    // 192 rows x 64 B
@@ -82,8 +89,9 @@ struct TLayout {
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;          // + 1024-B alignment slack
     // tensor memory: the accumulators (kTiles x NTOK columns) at column 0,
-    // then from column 128 SA A stages (kTiles x 32 columns each: 64 k of
-    // bf16 pairs)
+    // then from column 128 SA A stages (kTiles x kAK / 2 columns each: kAK k
+    // of bf16 pairs).  A stages of a whole group (two slots) measured ~3%
+    // faster than half-group stages (four slots): half the hand-offs.
     static constexpr int D_COLS = kTiles * NTOK;
     static constexpr int A_COL = 128;
     static constexpr int A_COLS = kTiles * (kAK / 2);
@@ -239,10 +247,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tc_fence_after();
 #pragma unroll
                         for (int ks = 0; ks < kAK / 16; ++ks) {
-                            // the descriptor's start address is in 16-byte units
+                            // k offset in the group -> x box (64 k) and 32-byte step
+                            // in it; the descriptor's start address is in 16-byte units
+                            const int kg = h * kAK + ks * 16;
                             tc_mma_ts(tmem + t * NTOK,
                                       tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
-                                      bdesc + static_cast<uint64_t>((h * L::X_BOX + ks * 32) >> 4),
+                                      bdesc + static_cast<uint64_t>(
+                                                  ((kg >> 6) * L::X_BOX + (kg & 63) * 2) >> 4),
                                       idesc, (g | h | ks) != 0);
                         }
                         issued = true;
@@ -319,11 +330,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t wrow = sbase + s * L::STAGE + row_off;
                 for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
                     const int a = ia % SA;
-                    uint4 c0 = make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
-                    uint4 c1 = c0;  // code 8 everywhere: rows past the range are zero
-                    if (valid) {
-                        c0 = lds128(wrow + 16u * ((2u * h) ^ swz));
-                        c1 = lds128(wrow + 16u * ((2u * h + 1u) ^ swz));
+                    // code 8 everywhere: rows past the range are zero
+                    uint4 c[kChunks];
+#pragma unroll
+                    for (int i = 0; i < kChunks; ++i) {
+                        c[i] = make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
+                        if (valid)
+                            c[i] = lds128(wrow + 16u * (static_cast<uint32_t>(kChunks * h + i) ^ swz));
                     }
                     if (!wait_warp(empty_a(t, a), ((ia / SA) & 1u) ^ 1u, abort_flag, p.status,
                                    p.wait_ns)) {
@@ -331,21 +344,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
-                    uint32_t v[32];
-                    codes_signed(c0.x, v + 0);
-                    codes_signed(c0.y, v + 4);
-                    codes_signed(c0.z, v + 8);
-                    codes_signed(c0.w, v + 12);
-                    codes_signed(c1.x, v + 16);
-                    codes_signed(c1.y, v + 20);
-                    codes_signed(c1.z, v + 24);
-                    codes_signed(c1.w, v + 28);
-                    // wd = RNE_bf16((q - 8) * s): the exact q - 8 times the scale, one rounding
+                    // per 32 codes: exact q - 8 pairs, then wd = RNE_bf16((q - 8) * s)
+                    // (one rounding), stored as 32 x 16 bf16 pairs of the row's lane
+                    const bool st_ok =
+                        dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (kAK / 2) <= L::TMEM_COLS,
+                                  p.status);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] = bf16x2_mul(v[j], s2);
-                    if (dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (kAK / 2) <= L::TMEM_COLS,
-                                  p.status))
-                        tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS + t * (kAK / 2), v);
+                    for (int i = 0; i < kChunks; i += 2) {
+                        uint32_t v[32];
+                        codes_signed(c[i].x, v + 0);
+                        codes_signed(c[i].y, v + 4);
+                        codes_signed(c[i].z, v + 8);
+                        codes_signed(c[i].w, v + 12);
+                        codes_signed(c[i + 1].x, v + 16);
+                        codes_signed(c[i + 1].y, v + 20);
+                        codes_signed(c[i + 1].z, v + 24);
+                        codes_signed(c[i + 1].w, v + 28);
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = bf16x2_mul(v[j], s2);
+                        if (st_ok)
+                            tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS +
+                                                   t * (kAK / 2) + i * 16,
+                                               v);
+                    }
                     tmem_st_wait();
                     tc_fence_before();
                     __syncwarp();
