@@ -149,3 +149,36 @@ def test_fused_gelu_bias_residual_in_place_fullsize_sampled():
     gotc = bf16_to_f64(res[:, torch.from_numpy(cols).cuda()])
     assert_close_fused(gotc, yc, refc, W.ACT_GELU, bias[cols], "gelu columns")
     assert W.get_device_error() == W.OK
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("M", [8, 24])
+def test_fused_swiglu_small_m_readout_scale(M):
+    """SwiGLU + bias + residual on the small-M streaming kernels (warp-level
+    at M = 8, tensor-core at M = 24) over the full gate/up weights (K 12288 x
+    2 x 49152 interleaved rows: more row chunks than SMs), on sampled output
+    columns for every token."""
+    W = _W()
+    c = S.MLP_SWIGLU
+    packed, scales, wd, sd = prepare_weights(c.N, c.K, c.g, c.w_seed)
+    x = S.make_x(M, c.K, 700 + M, "cuda")
+    n_out = c.N // 2
+    rng = np.random.default_rng(13 + M)
+    bf16 = lambda a: S.bf16_bits(torch.from_numpy(a.astype(np.float32)).to(torch.bfloat16))
+    bias = bf16(0.5 * rng.normal(size=c.N))
+    res = bf16(0.5 * rng.normal(size=(M, n_out)))
+    to_dev = lambda b: torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).cuda()
+    out = W.linear_fused(x, wd, sd, c.g, act=W.ACT_SWIGLU, bias=to_dev(bias), residual=to_dev(res))
+    torch.cuda.synchronize()
+    cols = {0, 161, 162, 191, 192, n_out // 3, n_out // 2 + 7, n_out - 1}
+    cols.update(int(v) for v in rng.integers(0, n_out, size=8))
+    cols = np.array(sorted(cols), dtype=np.int64)
+    wrows = np.stack([2 * cols, 2 * cols + 1], axis=1).ravel()      # (gate, up) per column
+    mi = np.repeat(np.arange(M, dtype=np.int64), len(wrows))
+    ni = np.tile(wrows, M)
+    y = O.linear_points(S.bf16_bits(x), packed, scales, c.N, c.K, c.g, mi, ni,
+                        nthreads=O.max_threads()).reshape(M, len(wrows))
+    ref = O.epilogue_rows(y, W.ACT_SWIGLU, bias=bias[wrows], residual=res[:, cols])
+    got = bf16_to_f64(out[:, torch.from_numpy(cols).cuda()])
+    assert_close_fused(got, y, ref, W.ACT_SWIGLU, bias[wrows], f"swiglu small M={M}")
+    assert W.get_device_error() == W.OK
