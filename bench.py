@@ -44,8 +44,14 @@ NCU_TRAFFIC = {
     ("stack", "ts", "99063559ec7b3d82"): 7.1207e9 * 4,
     # QKV prefill 4096x12288x36864 (256-token CTA pairs), one launch (full capture)
     ("qkv", "ts", "99063559ec7b3d82"): 1.2102e9 + 0.2921e9,
+    # MLP up / down at 8192 tokens (256-token CTA pairs), one launch each
+    # (DRAM counters only; profiles/gemm_pair_mlp_traffic_8192.md)
+    ("mlp_up", "ts", "99063559ec7b3d82"): 3.2250e9 + 0.7964e9,
+    ("mlp_down", "ts", "99063559ec7b3d82"): 5.5703e9 + 0.2024e9,
     # small-M readout, M = 8 (warp-level kernel), 12288x49152, one launch
     ("gemv", "gemv", "270f49f687deb1b3"): 0.31859e9 + 0.00380e9,
+    # the same at M = 16 (16 token columns), one launch (DRAM counters only)
+    ("gemv16", "gemv", "270f49f687deb1b3"): 0.31808e9 + 0.00319e9,
     # small-M readout, M = 32 (tensor-core kernel), 12288x49152, one launch
     ("gemv32", "gemvtc", "88cfd3cc92630dc4"): 0.32655e9 + 0.00339e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
@@ -77,8 +83,8 @@ def ncu_traffic(config: str, m: int, pairs: int = 8):
     if config == "gemv":
         if 17 <= m <= 32:  # the tensor-core kernel; the capture is of M = 32
             return NCU_TRAFFIC.get(("gemv32", "gemvtc", kernel_source_hash("gemvtc")))
-        if m > 8:  # the capture is of the M <= 8 instantiation
-            return None
+        if m > 8:  # the M = 9..16 instantiation, captured at M = 16
+            return NCU_TRAFFIC.get(("gemv16", "gemv", kernel_source_hash("gemv")))
         kind = "gemv"
     else:
         kind = "ts"
@@ -774,8 +780,8 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
         ach, peak, unit = wl.bytes / t / 1e9, peaks["hbm_gbs"], "GB/s"
     else:
         ach, peak, unit = wl.flops / t / 1e12, peaks["bf16_tflops"], "TFLOP/s"
-    traffic = (ncu_traffic("qkv", lc.M) if name == "qkv_prefill"
-               else ncu_traffic("gemv", lc.M) if hbm else None)
+    traffic = (ncu_traffic("gemv", lc.M) if hbm else
+               ncu_traffic({"qkv_prefill": "qkv"}.get(name, name), lc.M))
     res = {"workload": lc.name, "value": ach, "unit": unit, "us_per_launch": t * 1e6,
            "launches": steps,
            "us_per_launch_reps": {"reps": reps, "launches_per_rep": per_rep,
