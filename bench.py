@@ -738,19 +738,17 @@ def main():
     return 0
 
 
-def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
-    """One linear workload timed alone (CUDA events on the launching stream,
-    clocks sampled meanwhile), with its own roofline: TFLOP/s against the
-    measured bf16 burst peak for the GEMMs, GB/s against the measured copy
-    bandwidth for the small-M readout."""
+def _timed_reps(wl, gpu, warmup, seconds):
+    """Times wl.step() alone (CUDA events on the launching stream, clocks
+    sampled meanwhile): warm-up launches, the last two timed to size the timed
+    region at about `seconds` (so that the clock sampler sees it), then 10
+    back-to-back repetitions, each bracketed by its own events.  Returns the
+    mean time per launch over all of them, the launch count, and the
+    per-launch spread over the repetitions and the clock summary as dicts."""
     import torch
-    from paper_2608_30877_gb300 import w4a16 as W
-    wl = LinearWorkload(lc.name, lc.M, lc.N, lc.K, lc.g, lc.w_seed, copies)
     stream = torch.cuda.current_stream()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(gpu) as clk:
-        # warm-up launches, the last ones timed to size the timed region at
-        # about `seconds` (so that the clock sampler sees it)
         for _ in range(warmup - 2):
             wl.step()
         a.record(stream)
@@ -758,9 +756,6 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
             wl.step()
         b.record(stream)
         b.synchronize()
-        # the timed region as 10 back-to-back repetitions, each bracketed by
-        # its own events: the mean over all launches and the spread of the
-        # per-launch time over the repetitions
         reps = 10
         per_rep = max(1, int(seconds / (a.elapsed_time(b) / 2e3)) // reps)
         steps = reps * per_rep
@@ -773,29 +768,62 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
         ev[-1].synchronize()
     rep_us = sorted(ev[r].elapsed_time(ev[r + 1]) * 1e3 / per_rep for r in range(reps))
     t = ev[0].elapsed_time(ev[-1]) / 1e3 / steps
-    if W.get_device_error() != W.OK:
-        raise RuntimeError(f"device status word set during {name}")
-    hbm = lc.M <= 32
+    spread = {"reps": reps, "launches_per_rep": per_rep,
+              "median": (rep_us[reps // 2 - 1] + rep_us[reps // 2]) / 2,
+              "min": rep_us[0], "max": rep_us[-1]}
+    return t, steps, spread, clk.summary()
+
+
+def _config_line(workload, wl, t, steps, spread, clocks, peaks, hbm, traffic, l2):
     if hbm:
         ach, peak, unit = wl.bytes / t / 1e9, peaks["hbm_gbs"], "GB/s"
     else:
         ach, peak, unit = wl.flops / t / 1e12, peaks["bf16_tflops"], "TFLOP/s"
+    return {"workload": workload, "value": ach, "unit": unit, "us_per_launch": t * 1e6,
+            "launches": steps, "us_per_launch_reps": spread, "clocks": clocks,
+            "roofline": {"bound": "hbm" if hbm else "tensor", "achieved": ach, "peak": peak,
+                         "unit": unit, "frac": ach / peak,
+                         "frac_nominal": ach / (NOMINAL_HBM_GBS if hbm else NOMINAL_BF16_TFLOPS),
+                         "traffic": traffic,
+                         "peak_source": peaks["source"] + (" hbm_gbs" if hbm else " bf16_tflops"),
+                         "algorithmic_bytes": wl.bytes, "flops": wl.flops},
+            "l2": l2}
+
+
+def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=1.2):
+    """One linear workload timed alone, with its own roofline: TFLOP/s
+    against the measured bf16 burst peak for the GEMMs, GB/s against the
+    measured copy bandwidth for the small-M readout."""
+    import torch
+    from paper_2608_30877_gb300 import w4a16 as W
+    wl = LinearWorkload(lc.name, lc.M, lc.N, lc.K, lc.g, lc.w_seed, copies)
+    t, steps, spread, clocks = _timed_reps(wl, gpu, warmup, seconds)
+    if W.get_device_error() != W.OK:
+        raise RuntimeError(f"device status word set during {name}")
+    hbm = lc.M <= 32
     traffic = (ncu_traffic("gemv", lc.M) if hbm else
                ncu_traffic({"qkv_prefill": "qkv"}.get(name, name), lc.M))
-    res = {"workload": lc.name, "value": ach, "unit": unit, "us_per_launch": t * 1e6,
-           "launches": steps,
-           "us_per_launch_reps": {"reps": reps, "launches_per_rep": per_rep,
-                                  "median": (rep_us[reps // 2 - 1] + rep_us[reps // 2]) / 2,
-                                  "min": rep_us[0], "max": rep_us[-1]},
-           "clocks": clk.summary(),
-           "roofline": {"bound": "hbm" if hbm else "tensor", "achieved": ach, "peak": peak,
-                        "unit": unit, "frac": ach / peak,
-                        "frac_nominal": ach / (NOMINAL_HBM_GBS if hbm else NOMINAL_BF16_TFLOPS),
-                        "traffic": traffic,
-                        "peak_source": peaks["source"] + (" hbm_gbs" if hbm else " bf16_tflops"),
-                        "algorithmic_bytes": wl.bytes, "flops": wl.flops},
-           "l2": ("weights rotate over 2 copies larger than L2" if copies > 1
-                  else "inputs larger than L2; no flush")}
+    res = _config_line(lc.name, wl, t, steps, spread, clocks, peaks, hbm, traffic,
+                       "weights rotate over 2 copies larger than L2" if copies > 1
+                       else "inputs larger than L2; no flush")
+    del wl
+    torch.cuda.empty_cache()
+    return res
+
+
+def time_attention_config(peaks, gpu, pairs=64, seconds=1.2):
+    """One attention prefill layer over the packed batch (64 pairs x 1024
+    tokens, 96 heads of 128, causal, 32K window) timed alone: TFLOP/s against
+    the measured bf16 burst peak."""
+    import torch
+    from paper_2608_30877_gb300 import w4a16 as W
+    wl = AttentionWorkload(pairs, 1024, 96, 32768, 9)
+    t, steps, spread, clocks = _timed_reps(wl, gpu, 4, seconds)
+    if W.get_device_error() != W.OK:
+        raise RuntimeError("device status word set during attention")
+    res = _config_line(f"attention_prefill_{pairs}x1024_h96_w32768", wl, t, steps, spread,
+                       clocks, peaks, False, ncu_traffic("attention", 0, pairs),
+                       "qkv (4.8 GB at 64 pairs) larger than L2; no flush")
     del wl
     torch.cuda.empty_cache()
     return res
@@ -803,8 +831,9 @@ def time_linear_config(name, lc, peaks, gpu, warmup, copies=1, seconds=0.6):
 
 def configs_sweep(peaks, gpu):
     """The other named workloads, each timed alone after the stack: the
-    QKV prefill, the MLP up and down projections (tensor-bound) and the
-    small-M readout at M = 1, 8, 16, 32 (HBM-bound)."""
+    QKV prefill, the MLP up and down projections (tensor-bound), the small-M
+    readout at M = 1, 8, 16, 32 (HBM-bound) and one attention prefill layer
+    (tensor-bound)."""
     from paper_2608_30877_gb300 import synthetic as S
     out = {}
     for key, lc in (("qkv_prefill", S.QKV_PREFILL), ("mlp_up", S.MLP_UP),
@@ -813,6 +842,7 @@ def configs_sweep(peaks, gpu):
     for m in S.GEMV_MS:
         out[f"gemv_m{m}"] = time_linear_config(f"gemv_m{m}", S.gemv_case(m), peaks, gpu,
                                                warmup=6, copies=2)
+    out["attention_prefill"] = time_attention_config(peaks, gpu)
     return out
 
 
