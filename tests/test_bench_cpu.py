@@ -46,5 +46,11 @@ def test_attention_traffic_scales_with_pairs():
         return
     assert bench.ncu_traffic("attention", 0, 64) == t8 * 8
     assert bench.ncu_traffic("topk", 0) is None
-    # the small-M capture is of the M <= 8 instantiation only
-    assert bench.ncu_traffic("gemv", 16) is None
+    # M = 9..16 read the M = 16 capture, M = 17..32 the tensor-core kernel's
+    h = bench.kernel_source_hash("gemv")
+    assert bench.ncu_traffic("gemv", 12) == bench.NCU_TRAFFIC.get(("gemv16", "gemv", h))
+    assert bench.ncu_traffic("gemv", 3) == bench.NCU_TRAFFIC.get(("gemv", "gemv", h))
+    t = bench.kernel_source_hash("ts")
+    for c in ("mlp_up", "mlp_down", "qkv"):
+        assert bench.ncu_traffic(c, 8192) == bench.NCU_TRAFFIC.get((c, "ts", t))
+    assert bench.ncu_traffic("mlp_swiglu", 8192) is None
