@@ -53,7 +53,7 @@ NCU_TRAFFIC = {
     # the same at M = 16 (16 token columns), one launch (DRAM counters only)
     ("gemv16", "gemv", "270f49f687deb1b3"): 0.31808e9 + 0.00319e9,
     # small-M readout, M = 32 (tensor-core kernel), 12288x49152, one launch
-    ("gemv32", "gemvtc", "88cfd3cc92630dc4"): 0.32655e9 + 0.00339e9,
+    ("gemv32", "gemvtc", "b81ddd27f1e19156"): 0.32655e9 + 0.00362e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
     # one 8-pair launch); scaled by pairs / 8 for the benched launch
     ("attention", "attn", "3294a8d7153edae5"): 0.8125e9 + 0.1834e9,

@@ -78,10 +78,11 @@ typedef enum {
  *   w_packed_u8  [N, K/2] uint8, device, layout above
  *   scales_bf16  [N, K/g] bf16, device
  *   out_bf16     [M, N]   bf16, device, written in full
- * Dispatch: M > 32 runs the fused dequant + tcgen05 GEMM; M <= 32 with
- * g = 128 runs a bandwidth-bound row-range streaming kernel (warp-level
- * MMAs for M <= 16, tcgen05 for M = 17..32); other small M (g != 128) run
- * the tcgen05 GEMM with 32-token tiles.  The tcgen05 kernels multiply x by
+ * Dispatch: M > 128 runs the fused dequant + tcgen05 GEMM; M <= 128 with
+ * g = 128 runs a row-range streaming kernel that reads the weights once
+ * (warp-level MMAs for M <= 16, tcgen05 for M = 17..128); M <= 32 with
+ * g != 128 runs the tcgen05 GEMM with 32-token tiles, other M with g != 128
+ * the GEMM.  The tcgen05 kernels multiply x by
  * the dequantised weights wd defined above, so they differ from each other
  * only in the fp32 summation order.  The warp-level streaming kernel factors
  * the scale out of each group instead: it sums x * (code - 8) over the group

@@ -223,12 +223,12 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uin
     return r == CUDA_SUCCESS ? W4A16_OK : W4A16_ERR_CUDA;
 }
 
-// M <= 32 with g = 128: the streaming kernel (rows spread evenly over the
-// SMs).
+// M <= 128 with g = 128: the streaming kernels (rows spread evenly over the
+// SMs); the warp-level one takes at most 32 token columns.
 int launch_gemv(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                 int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
                 cudaStream_t stream) {
-    const bool tc = M >= g_small_m_tc_from;
+    const bool tc = M > 32 || M >= g_small_m_tc_from;
     const int T = tc ? gemv_tc_tokens(M) : gemv_tokens_per_tile(M);
     const int RB = tc ? gemv_tc_rows_per_cta(N, st.sm_count) : gemv_rows_per_cta(N, st.sm_count);
     alignas(64) CUtensorMap tx;
@@ -261,7 +261,10 @@ int launch_gemv(const DeviceState& st, const void* x, const void* w, const void*
 int launch_linear(const DeviceState& st, const void* x, const void* w, const void* s, void* out,
                   int64_t M, int64_t N, int64_t K, int64_t g, const Epilogue& epi,
                   cudaStream_t stream) {
-    if (M <= 32 && g == 128 && K % 128 == 0 && g_small_m_streaming)
+    // up to 128 tokens the weights stream once per call on the streaming
+    // tensor-core kernel (12288 x 49152: M = 64 103 us there against 212 on the
+    // 256-token GEMM tiles, M = 128 141 against 214)
+    if (M <= 128 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
     const TsVariant v = M <= 32                      ? TsVariant::kGemv32
                         : g_gemm_pair && M >= g_gemm_wide_from ? TsVariant::kGemmPairWide

@@ -1,6 +1,7 @@
-// Small-M (M <= 32, g = 128) int4-dequant + matmul on the 5th-generation
-// tensor core: the bandwidth-bound regime where the whole packed weight
-// matrix streams from HBM once per call.
+// Small-M (M <= 128, g = 128) int4-dequant + matmul on the 5th-generation
+// tensor core: the regime where the whole packed weight matrix streams from
+// HBM once per call (the GEMM's 256-token tiles would leave most of their
+// columns empty and split the weight rows unevenly over the SMs).
 //
 // out[m, n] = sum_k x[m, k] * wd[n, k],   wd = RNE_bf16((q[n, k] - 8) * s[n, k / g])
 //
@@ -15,7 +16,8 @@
 //
 // Per CTA (persistent, one per SM): a contiguous range of RB <= 384 weight
 // rows (RB = N / #SMs rounded up to even), as three MMA tiles of 128 rows,
-// each with ONE fp32 accumulator in tensor memory for the whole K walk.
+// each with ONE fp32 accumulator of NTOK = 16, 32, 64 or 128 token columns in
+// tensor memory for the whole K walk.
 // Per scale group of 128 k:
 //   warp 0      TMA: two 64-k boxes of x (NTOK token rows, 128-byte swizzle,
 //               rows >= M zero-filled) and two boxes of RB/2 rows x 64 B of
@@ -28,7 +30,8 @@
 //               multiply per pair) -> tcgen05.st into a ring of SA A stages
 //               (one per group);
 //               after the last group, the epilogue: tcgen05.ld of the row's
-//               NTOK accumulators, then the (fused) epilogue from registers;
+//               NTOK accumulators in slices of up to 32, each slice's (fused)
+//               epilogue from registers;
 //   warps 1, 3, 16  one thread each, one per tile, issues
 //               D_t[128 x NTOK] += A_t[128 x 16] x B[NTOK x 16]^T (A from
 //               tensor memory, B = x in shared memory), 8 MMAs per group,
@@ -51,17 +54,10 @@ namespace w4a16 {
 
 namespace {
 
-constexpr int kTiles = 3;                 // MMA tiles of 128 rows per CTA
-constexpr int kRowsMax = 128 * kTiles;    // rows per CTA chunk
+constexpr int kTilesMax = 3;              // MMA tiles of 128 rows per CTA, at most
 constexpr int kGroupK = 128;              // k per TMA stage = one scale group
-#ifndef W4A16_TC_AK
-#define W4A16_TC_AK 128
-#endif
-constexpr int kAK = W4A16_TC_AK;          // k per tensor-memory A stage (64 or 128)
-static_assert(kAK == 64 || kAK == 128, "A stages of half or whole scale groups");
-constexpr int kChunks = kAK / 32;         // 16-byte chunks (32 codes) per row and A stage
 constexpr int kFirstRowWarp = 4;          // warps 4..15 (warp % 4 = TMEM sub-partition)
-constexpr int kRowWarps = 4 * kTiles;     // dequant + epilogue warps
+constexpr int kRowWarps = 4 * kTilesMax;  // dequant + epilogue warps
 constexpr int kLastIssuerWarp = kFirstRowWarp + kRowWarps;  // warp 16: tile 2's MMAs
 constexpr int kThreads = 32 * (kLastIssuerWarp + 1);
 
@@ -70,31 +66,52 @@ __device__ __forceinline__ int issuer_tile(int warp) {
     return warp == 1 ? 0 : warp == 3 ? 1 : warp == kLastIssuerWarp ? 2 : -1;
 }
 
+// 32 lanes x 16 columns of 32 bits (see tmem_st_32x32b_x32).
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t* v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15])
+        : "memory");
+}
+
 template <int NTOK>
 struct TLayout {
-    static_assert(NTOK == 16 || NTOK == 32, "MMA N for M = 128");
-    static constexpr int S = NTOK == 32 ? 6 : 7;                     // TMA stage slots
+    static_assert(NTOK == 16 || NTOK == 32 || NTOK == 64 || NTOK == 128, "MMA N for M = 128");
+    // MMA tiles of 128 rows per CTA (with 128 tokens, two tiles and 256 rows
+    // per CTA would leave room for more A stages but need a second wave of
+    // chunks at N = 49152: 207 against 141 us)
+    static constexpr int TILES = kTilesMax;
+    static constexpr int ROWS_MAX = 128 * TILES;                     // rows per CTA chunk
+    static constexpr int S = NTOK == 128 ? 3 : NTOK == 64 ? 5 : NTOK == 32 ? 6 : 7;  // TMA slots
+    // k per tensor-memory A stage: a whole scale group; half of one where the
+    // 64-token accumulators leave room for three half-group slots only; a
+    // quarter where the 128-token accumulators leave room for two
+    static constexpr int AK = NTOK == 128 ? 32 : NTOK == 64 ? 64 : 128;
+    static constexpr int CHUNKS = AK / 32;  // 16-byte chunks (32 codes) per row and A stage
     // A stage slots: as many as fit next to the accumulators
-    static constexpr int SA = kAK == 64 ? 4 : 2;
+    static constexpr int SA = NTOK == 64 ? 3 : 2;
     static constexpr int X_BOX = NTOK * 128;                         // 64 k x NTOK tokens
     static constexpr int X_BYTES = 2 * X_BOX;
-    static constexpr int W_HALF = (kRowsMax / 2) * (kGroupK / 2);    // 192 rows x 64 B
+    static constexpr int W_HALF = (ROWS_MAX / 2) * (kGroupK / 2);    // ROWS_MAX / 2 rows x 64 B
     static constexpr int W_BYTES = 2 * W_HALF;
     static constexpr int STAGE = X_BYTES + W_BYTES;                  // x, then the weights
     // full_tma[S], empty_smem[S], x_ready[S], then per tile: full_a[SA],
     // empty_a[SA], d_full, d_empty, drain
     static constexpr int BAR_OFF = S * STAGE;
     static constexpr int TILE_BARS = 2 * SA + 3;
-    static constexpr int NBARS = 3 * S + kTiles * TILE_BARS;
+    static constexpr int NBARS = 3 * S + TILES * TILE_BARS;
     static constexpr int MISC_OFF = BAR_OFF + NBARS * 8;
     static constexpr int SMEM_BYTES = MISC_OFF + 16 + 1024;          // + 1024-B alignment slack
-    // tensor memory: the accumulators (kTiles x NTOK columns) at column 0,
-    // then from column 128 SA A stages (kTiles x kAK / 2 columns each: kAK k
+    // tensor memory: the accumulators (TILES x NTOK columns) at column 0,
+    // then from column A_COL SA A stages (TILES x AK / 2 columns each: AK k
     // of bf16 pairs).  A stages of a whole group (two slots) measured ~3%
     // faster than half-group stages (four slots): half the hand-offs.
-    static constexpr int D_COLS = kTiles * NTOK;
-    static constexpr int A_COL = 128;
-    static constexpr int A_COLS = kTiles * (kAK / 2);
+    static constexpr int D_COLS = TILES * NTOK;
+    static constexpr int A_COL = NTOK == 128 ? 384 : NTOK == 64 ? 192 : 128;
+    static constexpr int A_COLS = TILES * (AK / 2);
     static constexpr int TMEM_COLS = 512;
     static_assert(D_COLS <= A_COL && A_COL + SA * A_COLS <= TMEM_COLS,
                   "tensor memory holds 512 columns");
@@ -139,7 +156,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(empty_smem(s), 5 * p.nt);
             mbar_init(x_ready(s), 1);
         }
-        for (int t = 0; t < kTiles; ++t) {
+        for (int t = 0; t < L::TILES; ++t) {
             for (int a = 0; a < SA; ++a) {
                 mbar_init(full_a(t, a), 4);  // the tile's four row warps
                 mbar_init(empty_a(t, a), 1);
@@ -216,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ MMA issuers
         // (tiles past the chunk's rows, t >= p.nt, are not computed)
         const int t = issuer_tile(warp);
-        if (lane == 0 && t < p.nt) {
+        if (lane == 0 && t < p.nt && t < L::TILES) {
             constexpr uint32_t idesc = idesc_bf16_f32(128, NTOK);
             uint32_t it = 0, ia = 0, nchunk = 0;
             bool ok = true, issued = false;
@@ -237,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_fence_after();
                     const uint64_t bdesc = sdesc_kmajor_sw128(sbase + s * L::STAGE);
-                    for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
+                    for (int h = 0; h < kGroupK / L::AK; ++h, ++ia) {
                         const int a = ia % SA;
                         if (!wait_one(full_a(t, a), (ia / SA) & 1u, abort_flag, p.status,
                                       p.wait_ns)) {
@@ -246,12 +263,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         tc_fence_after();
 #pragma unroll
-                        for (int ks = 0; ks < kAK / 16; ++ks) {
+                        for (int ks = 0; ks < L::AK / 16; ++ks) {
                             // k offset in the group -> x box (64 k) and 32-byte step
                             // in it; the descriptor's start address is in 16-byte units
-                            const int kg = h * kAK + ks * 16;
+                            const int kg = h * L::AK + ks * 16;
                             tc_mma_ts(tmem + t * NTOK,
-                                      tmem + L::A_COL + a * L::A_COLS + t * (kAK / 2) + ks * 8,
+                                      tmem + L::A_COL + a * L::A_COLS + t * (L::AK / 2) + ks * 8,
                                       bdesc + static_cast<uint64_t>(
                                                   ((kg >> 6) * L::X_BOX + (kg & 63) * 2) >> 4),
                                       idesc, (g | h | ks) != 0);
@@ -297,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else if (warp >= kFirstRowWarp && warp < kLastIssuerWarp &&
-               (warp - kFirstRowWarp) / 4 < p.nt) {
+               (warp - kFirstRowWarp) / 4 < p.nt && (warp - kFirstRowWarp) / 4 < L::TILES) {
         // ------------------------------------------------------------ dequant + epilogue
         const int t = (warp - kFirstRowWarp) >> 2;  // MMA tile
         const int sub = warp & 3;                   // TMEM sub-partition
@@ -328,15 +345,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 const uint32_t wrow = sbase + s * L::STAGE + row_off;
-                for (int h = 0; h < kGroupK / kAK; ++h, ++ia) {
+                for (int h = 0; h < kGroupK / L::AK; ++h, ++ia) {
                     const int a = ia % SA;
                     // code 8 everywhere: rows past the range are zero
-                    uint4 c[kChunks];
+                    uint4 c[L::CHUNKS];
 #pragma unroll
-                    for (int i = 0; i < kChunks; ++i) {
+                    for (int i = 0; i < L::CHUNKS; ++i) {
                         c[i] = make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
                         if (valid)
-                            c[i] = lds128(wrow + 16u * (static_cast<uint32_t>(kChunks * h + i) ^ swz));
+                            c[i] = lds128(wrow + 16u * (static_cast<uint32_t>(L::CHUNKS * h + i) ^ swz));
                     }
                     if (!wait_warp(empty_a(t, a), ((ia / SA) & 1u) ^ 1u, abort_flag, p.status,
                                    p.wait_ns)) {
@@ -347,25 +364,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // per 32 codes: exact q - 8 pairs, then wd = RNE_bf16((q - 8) * s)
                     // (one rounding), stored as 32 x 16 bf16 pairs of the row's lane
                     const bool st_ok =
-                        dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (kAK / 2) <= L::TMEM_COLS,
+                        dbg_check(L::A_COL + a * L::A_COLS + (t + 1) * (L::AK / 2) <= L::TMEM_COLS,
                                   p.status);
+                    if constexpr (L::CHUNKS == 1) {
+                        uint32_t v[16];
+                        codes_signed(c[0].x, v + 0);
+                        codes_signed(c[0].y, v + 4);
+                        codes_signed(c[0].z, v + 8);
+                        codes_signed(c[0].w, v + 12);
 #pragma unroll
-                    for (int i = 0; i < kChunks; i += 2) {
-                        uint32_t v[32];
-                        codes_signed(c[i].x, v + 0);
-                        codes_signed(c[i].y, v + 4);
-                        codes_signed(c[i].z, v + 8);
-                        codes_signed(c[i].w, v + 12);
-                        codes_signed(c[i + 1].x, v + 16);
-                        codes_signed(c[i + 1].y, v + 20);
-                        codes_signed(c[i + 1].z, v + 24);
-                        codes_signed(c[i + 1].w, v + 28);
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) v[j] = bf16x2_mul(v[j], s2);
+                        for (int j = 0; j < 16; ++j) v[j] = bf16x2_mul(v[j], s2);
                         if (st_ok)
-                            tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS +
-                                                   t * (kAK / 2) + i * 16,
+                            tmem_st_32x32b_x16(lane_base + L::A_COL + a * L::A_COLS + t * (L::AK / 2),
                                                v);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < L::CHUNKS; i += 2) {
+                            uint32_t v[32];
+                            codes_signed(c[i].x, v + 0);
+                            codes_signed(c[i].y, v + 4);
+                            codes_signed(c[i].z, v + 8);
+                            codes_signed(c[i].w, v + 12);
+                            codes_signed(c[i + 1].x, v + 16);
+                            codes_signed(c[i + 1].y, v + 20);
+                            codes_signed(c[i + 1].z, v + 24);
+                            codes_signed(c[i + 1].w, v + 28);
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) v[j] = bf16x2_mul(v[j], s2);
+                            if (st_ok)
+                                tmem_st_32x32b_x32(lane_base + L::A_COL + a * L::A_COLS +
+                                                       t * (L::AK / 2) + i * 16,
+                                                   v);
+                        }
                     }
                     tmem_st_wait();
                     tc_fence_before();
@@ -383,47 +413,57 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            float acc[NTOK];
+            // the row's accumulators in slices of EC tokens (registers), then
+            // the (fused) epilogue of each slice
+            constexpr int EC = NTOK < 32 ? NTOK : 32;
+            const Epilogue& ep = p.epi;
+            // SwiGLU pairs rows (n, n ^ 1) = (gate, up): RB is even, so n has
+            // the parity of its lane and the partner is lane ^ 1
+            const float bias =
+                (FUSED && ep.bias != nullptr && valid) ? bf16_to_f32(ep.bias[n]) : 0.0f;
+#pragma unroll 1
+            for (int m0 = 0; m0 < NTOK; m0 += EC) {
+                float acc[EC];
 #pragma unroll
-            for (int half = 0; half < NTOK / 16; ++half) {
-                uint32_t d[16];
-                tmem_ld_32x32b_x16(lane_base + t * NTOK + half * 16, d);
-                tmem_ld_wait_x16(d);
+                for (int half = 0; half < EC / 16; ++half) {
+                    uint32_t d[16];
+                    tmem_ld_32x32b_x16(lane_base + t * NTOK + m0 + half * 16, d);
+                    tmem_ld_wait_x16(d);
 #pragma unroll
-                for (int j = 0; j < 16; ++j) acc[half * 16 + j] = __uint_as_float(d[j]);
+                    for (int j = 0; j < 16; ++j) acc[half * 16 + j] = __uint_as_float(d[j]);
+                }
+                if constexpr (!FUSED) {
+#pragma unroll
+                    for (int j = 0; j < EC; ++j) {
+                        const int m = m0 + j;
+                        if (valid && m < p.M)
+                            p.out[static_cast<int64_t>(m) * p.N + n] = f32_to_bf16_rn(acc[j]);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < EC; ++j) {
+                        const int m = m0 + j;
+                        const float z = acc[j] + bias;
+                        if (ep.act == kActSwiGLU) {
+                            const float up = __shfl_xor_sync(0xffffffffu, z, 1);
+                            if ((lane & 1) == 0 && valid && m < p.M) {
+                                const int64_t o = static_cast<int64_t>(m) * ep.n_out + (n >> 1);
+                                float h = silu_f32(z) * up;
+                                if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                                p.out[o] = f32_to_bf16_rn(h);
+                            }
+                        } else if (valid && m < p.M) {
+                            const int64_t o = static_cast<int64_t>(m) * ep.n_out + n;
+                            float h = ep.act == kActGELU ? gelu_f32(z) : z;
+                            if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
+                            p.out[o] = f32_to_bf16_rn(h);
+                        }
+                    }
+                }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(d_empty(t));  // the next chunk's MMAs may overwrite D
-            const Epilogue& ep = p.epi;
-            if constexpr (!FUSED) {
-#pragma unroll
-                for (int m = 0; m < NTOK; ++m)
-                    if (valid && m < p.M)
-                        p.out[static_cast<int64_t>(m) * p.N + n] = f32_to_bf16_rn(acc[m]);
-            } else {
-                // SwiGLU pairs rows (n, n ^ 1) = (gate, up): RB is even, so n
-                // has the parity of its lane and the partner is lane ^ 1
-                const float bias = (ep.bias != nullptr && valid) ? bf16_to_f32(ep.bias[n]) : 0.0f;
-#pragma unroll
-                for (int m = 0; m < NTOK; ++m) {
-                    const float z = acc[m] + bias;
-                    if (ep.act == kActSwiGLU) {
-                        const float up = __shfl_xor_sync(0xffffffffu, z, 1);
-                        if ((lane & 1) == 0 && valid && m < p.M) {
-                            const int64_t o = static_cast<int64_t>(m) * ep.n_out + (n >> 1);
-                            float h = silu_f32(z) * up;
-                            if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
-                            p.out[o] = f32_to_bf16_rn(h);
-                        }
-                    } else if (valid && m < p.M) {
-                        const int64_t o = static_cast<int64_t>(m) * ep.n_out + n;
-                        float h = ep.act == kActGELU ? gelu_f32(z) : z;
-                        if (ep.residual != nullptr) h += bf16_to_f32(ep.residual[o]);
-                        p.out[o] = f32_to_bf16_rn(h);
-                    }
-                }
-            }
         }
     }
 
@@ -453,18 +493,20 @@ cudaError_t launch_tc_variant(const CUtensorMap* tx, const CUtensorMap* tw, cons
 int gemv_tc_rows_per_cta(int64_t N, int sm_count) {
     int64_t per = (N + sm_count - 1) / sm_count;
     per = (per + 1) / 2 * 2;
-    if (per > kRowsMax) per = kRowsMax;
+    if (per > 128 * kTilesMax) per = 128 * kTilesMax;
     if (per < 2) per = 2;
     return static_cast<int>(per);
 }
 
-int gemv_tc_tokens(int64_t M) { return M <= 16 ? 16 : 32; }
+int gemv_tc_tokens(int64_t M) { return M <= 16 ? 16 : M <= 32 ? 32 : M <= 64 ? 64 : 128; }
 
 cudaError_t gemv_tc_launch(const CUtensorMap* tx, const CUtensorMap* tw, const GemvParams& p,
                            int sm_count, cudaStream_t stream) {
     const int grid = p.num_chunks < sm_count ? p.num_chunks : sm_count;
     if (p.M <= 16) return launch_tc_variant<16>(tx, tw, p, grid, stream);
-    return launch_tc_variant<32>(tx, tw, p, grid, stream);
+    if (p.M <= 32) return launch_tc_variant<32>(tx, tw, p, grid, stream);
+    if (p.M <= 64) return launch_tc_variant<64>(tx, tw, p, grid, stream);
+    return launch_tc_variant<128>(tx, tw, p, grid, stream);
 }
 
 }  // namespace w4a16

@@ -72,8 +72,9 @@ def short_waits():
 
 # (M, N, K, g): large-M tcgen05 GEMM on CTA pairs (several tiles per pair),
 # the warp-level small-M streaming kernel, the tcgen05 small-M streaming
-# kernel, the 32-token tcgen05 tiles (g = 64)
+# kernel with 32, 64 and 128 token columns, the 32-token tcgen05 tiles (g = 64)
 ABORT_CASES = [(600, 128 * 400, 2048, 128), (8, 8192, 4096, 128), (24, 8192, 4096, 128),
+               (48, 8192, 4096, 128), (96, 8192, 4096, 128),
                (16, 4096, 1024, 64)]
 
 
@@ -86,7 +87,7 @@ def test_linear_abort_path_under_short_waits(short_waits, M, N, K, g):
     W.linear(x, w, s, g)
     assert W.get_device_error() == W.ERR_TIMEOUT
     W.set_wait_limit(0)
-    _linear_still_correct(M=M if M <= 32 else 40, g=g)
+    _linear_still_correct(M=M if M <= 128 else 200, g=g)
 
 
 def test_fused_abort_path_under_short_waits(short_waits):

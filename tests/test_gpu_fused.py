@@ -36,7 +36,8 @@ def _case(M, N, K, g, seed, act, with_bias, with_res):
 
 SHAPES = [  # (M, N, K, g): streaming kernel, 32-token tcgen05 tiles, large-M GEMM
     (8, 1000, 1024, 128), (16, 4096, 512, 128), (24, 1234, 384, 128), (5, 200, 256, 64),
-    (300, 1000, 1024, 128), (40, 258, 512, 128),
+    (300, 1000, 1024, 128), (40, 258, 512, 128), (64, 1000, 1024, 128),
+    (100, 1000, 1024, 128),
 ]
 
 

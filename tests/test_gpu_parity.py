@@ -106,10 +106,10 @@ def test_linear_ragged_shapes(M, N, K, g):
 def test_linear_m_sweep_around_dispatch_threshold():
     W = _W()
     N, K, g = 256, 512, 128
-    x, xb, packed, scales = host_case(40, N, K, g, 77, 78)
+    x, xb, packed, scales = host_case(134, N, K, g, 77, 78)
     xd, wd, sd = to_device(x, packed, scales)
     ref = O.linear_rows(xb, packed, scales, N, K, g, nthreads=O.max_threads())
-    for M in range(1, 41):
+    for M in range(1, 135):
         out = W.linear(xd[:M].contiguous(), wd, sd, g)
         assert_close(bf16_to_f64(out), ref[:M], f"M={M}")
 
@@ -184,11 +184,13 @@ def test_error_codes_launch_nothing():
     (1, 1, 128, 128), (3, 100, 256, 128), (8, 1000, 1024, 128), (16, 4096, 512, 128),
     (17, 1234, 384, 128), (32, 8192, 256, 64), (32, 50000, 128, 128), (9, 77, 2048, 256),
     (8, 60000, 640, 128), (24, 60000, 1152, 128), (2, 53600, 2176, 128),
-    (20, 1, 128, 128), (29, 130, 128, 128),
+    (20, 1, 128, 128), (29, 130, 128, 128), (33, 130, 384, 128), (48, 60010, 256, 128),
+    (64, 1, 128, 128), (64, 4100, 1152, 128), (100, 60010, 256, 128), (128, 1, 128, 128),
+    (72, 4100, 1152, 128),
 ])
 def test_small_m_streaming_kernel_shapes(M, N, K, g):
-    """M <= 32 with g = 128 runs the row-range streaming kernel: ragged row
-    ranges, 8, 16 and 32 token columns, group counts that leave padding stages
+    """M <= 128 with g = 128 runs a row-range streaming kernel: ragged row
+    ranges, 8 to 128 token columns, group counts that leave padding stages
     in the last round of stage slots, and N large enough that a CTA takes a
     second row range (more row ranges than SMs)."""
     gpu, ref = _run_linear(M, N, K, g, seed=3 * M + N)
@@ -223,7 +225,9 @@ def test_small_m_kernels_every_m(kernel):
     import subprocess
     import sys
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    cases = [(M, 1000 + 2 * M, 384 if M % 2 else 1280) for M in (1, 2, 5, 8, 13, 16, 17, 24, 31, 32)]
+    Ms = (1, 2, 5, 8, 13, 16, 17, 24, 31, 32) + ((33, 40, 57, 64, 65, 99, 128) if kernel == "tc"
+                                                 else ())
+    cases = [(M, 1000 + 2 * M, 384 if M % 2 else 1280) for M in Ms]
     env = dict(os.environ, W4A16_SMALL_M=kernel)
     r = subprocess.run([sys.executable, "-c", _FORCED_KERNEL_CHECK.format(root=root, cases=cases)],
                        env=env, capture_output=True, text=True, timeout=600)
@@ -241,7 +245,7 @@ def test_small_m_kernels_several_chunks_per_cta(kernel):
     import subprocess
     import sys
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    cases = [(M, 60010, 256) for M in (3, 16, 24, 32)]
+    cases = [(M, 60010, 256) for M in (3, 16, 24, 32) + ((40, 64, 96, 128) if kernel == "tc" else ())]
     env = dict(os.environ, W4A16_SMALL_M=kernel)
     r = subprocess.run([sys.executable, "-c", _FORCED_KERNEL_CHECK.format(root=root, cases=cases)],
                        env=env, capture_output=True, text=True, timeout=600)
