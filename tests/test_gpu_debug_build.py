@@ -22,9 +22,11 @@ from paper_2608_30877_gb300 import w4a16 as W
 from tests.gpu_helpers import assert_close, bf16_to_f64, host_case, to_device
 assert W.LIB_PATH.endswith("libw4a16_debug.so"), W.LIB_PATH
 # (M, N, K, g): CTA-pair GEMM with a ragged last pair, warp-level and
-# tensor-core small-M kernels, 32-token tiles (g = 64)
+# tensor-core small-M kernels (32, 64 and 128 token columns), 32-token tiles
+# (g = 64)
 for (M, N, K, g) in [(300, 1000, 1024, 128), (520, 384, 512, 128), (8, 2000, 1280, 128),
-                     (24, 1234, 640, 128), (5, 200, 256, 64)]:
+                     (24, 1234, 640, 128), (48, 1234, 640, 128), (100, 1234, 640, 128),
+                     (5, 200, 256, 64)]:
     x, xb, packed, scales = host_case(M, N, K, g, M + 1, N + 2)
     xd, wd, sd = to_device(x, packed, scales)
     out = W.linear(xd, wd, sd, g)
