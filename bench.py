@@ -41,13 +41,14 @@ NCU_TRAFFIC = {
     # mean of one launch per stack shape at M = 16384 (384-token tiles, as in
     # the benched stack), scaled by 4 to M = 65536
     # (profiles/gemm_pair_wide_stack_traffic_m16384.md)
-    ("stack", "ts", "99063559ec7b3d82"): 7.1207e9 * 4,
-    # QKV prefill 4096x12288x36864 (256-token CTA pairs), one launch (full capture)
-    ("qkv", "ts", "99063559ec7b3d82"): 1.2102e9 + 0.2921e9,
-    # MLP up / down at 8192 tokens (256-token CTA pairs), one launch each
+    ("stack", "ts", "cc26b2d7ce6a2d19"): 7.1208e9 * 4,
+    # QKV prefill 4096x12288x36864 (384-token CTA pairs), one launch
+    # (profiles/gemm_pair_wide_qkv_prefill_4096x12288x36864.md)
+    ("qkv", "ts", "cc26b2d7ce6a2d19"): 1.4663e9 + 0.2894e9,
+    # MLP up / down at 8192 tokens (384-token CTA pairs), one launch each
     # (DRAM counters only; profiles/gemm_pair_mlp_traffic_8192.md)
-    ("mlp_up", "ts", "99063559ec7b3d82"): 3.2250e9 + 0.7964e9,
-    ("mlp_down", "ts", "99063559ec7b3d82"): 5.5703e9 + 0.2024e9,
+    ("mlp_up", "ts", "cc26b2d7ce6a2d19"): 3.9122e9 + 0.8025e9,
+    ("mlp_down", "ts", "cc26b2d7ce6a2d19"): 4.7823e9 + 0.1976e9,
     # small-M readout, M = 8 (warp-level kernel), 12288x49152, one launch
     ("gemv", "gemv", "270f49f687deb1b3"): 0.31859e9 + 0.00380e9,
     # the same at M = 16 (16 token columns), one launch (DRAM counters only)

@@ -81,11 +81,13 @@ bool g_small_m_streaming = true;
 // W4A16_SMALL_M=mma / tc forces one of them.
 int g_small_m_tc_from = 17;
 bool g_gemm_pair = true;  // large M on CTA pairs (cta_group::2); W4A16_GEMM_PAIR=0: one CTA per tile
-// CTA pairs with 384-token tiles from this many tokens on (the tile padding
-// is then under 2.4%): one dequantised weight stage serves 1.5x the tokens,
-// which under the power cap is 4.51 against 4.32 scored pairs/s on the stack.
-// W4A16_GEMM_WIDE=1 / 0 forces them on or off.
-int64_t g_gemm_wide_from = 16384;
+// CTA pairs with 384-token tiles (one dequantised weight stage serves 1.5x the
+// tokens) where they take fewer unit-costs per pair than the 256-token tiles
+// (ts_prefer_wide: tile padding and the last wave; 12288 x 49152: M = 4096
+// 2996 against 3135 us, M = 8192 MLP projections +7%, the stack 4.51 against
+// 4.32 scored pairs/s).  W4A16_GEMM_WIDE=1 / 0 forces them on or off (from this
+// many tokens on; -1: chosen per call).
+int64_t g_gemm_wide_from = -1;
 // barrier-wait limit of the launches (test hook w4a16_selftest_set_wait_limit)
 std::atomic<uint64_t> g_wait_limit_ns{kWaitLimitNs};
 
@@ -267,7 +269,10 @@ int launch_linear(const DeviceState& st, const void* x, const void* w, const voi
     if (M <= 128 && g == 128 && K % 128 == 0 && g_small_m_streaming)
         return launch_gemv(st, x, w, s, out, M, N, K, g, epi, stream);
     const TsVariant v = M <= 32                      ? TsVariant::kGemv32
-                        : g_gemm_pair && M >= g_gemm_wide_from ? TsVariant::kGemmPairWide
+                        : g_gemm_pair && (g_gemm_wide_from >= 0
+                                              ? M >= g_gemm_wide_from
+                                              : ts_prefer_wide(M, N, st.sm_count))
+                            ? TsVariant::kGemmPairWide
                         : g_gemm_pair                ? TsVariant::kGemmPair
                                                      : TsVariant::kGemm256;
     const int T = ts_tokens_per_tile(v);

@@ -47,6 +47,9 @@ int ts_tokens_per_tile(TsVariant v);
 int ts_x_box_tokens(TsVariant v);
 // Fills the grid size to use for the given problem (persistent or not).
 int ts_grid(TsVariant v, const TsParams& p, int sm_count);
+// Whether the 384-token CTA-pair tiles take fewer unit-costs per pair than the
+// 256-token ones for an M x N product (tile padding and the last wave).
+bool ts_prefer_wide(int64_t M, int64_t N, int sm_count);
 cudaError_t ts_launch(TsVariant v, const CUtensorMap* tmap_x, const CUtensorMap* tmap_w,
                       const TsParams& p, int grid, cudaStream_t stream);
 

@@ -729,6 +729,18 @@ int ts_x_box_tokens(TsVariant v) {
     return ts_tokens_per_tile(v);
 }
 
+bool ts_prefer_wide(int64_t M, int64_t N, int sm_count) {
+    // Each CTA pair walks ceil(units / pairs) units of (token tile, 256 weight
+    // rows); a unit of the 384-token tiles costs ~1.37 of a 256-token one
+    // (measured: 1.35-1.37 on the 4096- and 8192-token projections, 1.39 for
+    // one tile of each).  The tiles that give the fewer unit-costs per pair win.
+    const int64_t pairs = pair_slots(sm_count);
+    const int64_t per_tile = (N + 255) / 256;
+    const int64_t w256 = ((M + kGemmT - 1) / kGemmT * per_tile + pairs - 1) / pairs;
+    const int64_t w384 = ((M + kWideT - 1) / kWideT * per_tile + pairs - 1) / pairs;
+    return w384 * 137 < w256 * 100;
+}
+
 int ts_grid(TsVariant v, const TsParams& p, int sm_count) {
     if (v == TsVariant::kGemm256) return p.num_tiles < sm_count ? p.num_tiles : sm_count;
     if (v == TsVariant::kGemmPair || v == TsVariant::kGemmPairWide) {
