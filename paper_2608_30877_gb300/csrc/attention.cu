@@ -43,8 +43,10 @@ namespace {
 constexpr int kD = 128;        // head dimension
 constexpr int kBQ = 128;       // queries per job (MMA M)
 constexpr int kBKV = 64;       // keys per block (MMA N of S, K of PV)
-constexpr int kPvWarp = 6;
-constexpr int kThreads = 7 * 32;  // TMA warp, S-MMA warp, 4 softmax warps, PV-MMA warp
+constexpr int kPvWarp = 2;
+constexpr int kFirstSoftmaxWarp = 3;  // warps 3..10: two per TMEM sub-partition (warp % 4)
+constexpr int kSoftmaxWarps = 8;
+constexpr int kThreads = (kFirstSoftmaxWarp + kSoftmaxWarps) * 32;  // + TMA, S-MMA, PV-MMA warps
 
 struct AttnLayout {
     static constexpr int QBOX = kBQ * 128;    // one [128 rows x 64 cols] bf16 box: 16 KB
@@ -54,10 +56,10 @@ struct AttnLayout {
     static constexpr int Q_OFF = 0;
     static constexpr int K_OFF = Q_OFF + Q_TILE;       // two stages
     static constexpr int V_OFF = K_OFF + 2 * KV_TILE;  // two stages
-    // epilogue staging: per softmax warp 32 rows x 32 columns of bf16 output
+    // epilogue staging: per softmax warp 16 rows x 32 columns of bf16 output
     static constexpr int STAGE_OFF = V_OFF + 2 * KV_TILE;
-    static constexpr int STAGE_WARP = 32 * 64;
-    static constexpr int BAR_OFF = STAGE_OFF + 4 * STAGE_WARP;
+    static constexpr int STAGE_WARP = 16 * 64;
+    static constexpr int BAR_OFF = STAGE_OFF + kSoftmaxWarps * STAGE_WARP;
     // q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2],
     // s_full[2], p_full[2], o_ready[2], drain[2]
     static constexpr int NBARS = 18;
@@ -106,6 +108,65 @@ __device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_
         "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
         "r"(v[15])
         : "memory");
+}
+
+// 16-lane tensor-memory shapes (the warp covers 16 lanes from the address's
+// lane; thread t = 4 g + c).  16x256b.xN: register 4j + {0, 1} holds lane g,
+// columns 8j + 2c + {0, 1}; 4j + {2, 3} the same columns of lane g + 8.
+// 16x128b.xN: register 2j holds lane g, column 4j + c; 2j + 1 lane g + 8.
+__device__ __forceinline__ void tmem_ld_16x256b_x8(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x256b.x8.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, "
+        "[%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+          "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),
+          "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+          "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),
+          "=r"(v[31])
+        : "r"(taddr)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld_16x256b_x4(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+          "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_16x256b_x4(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x256b.x4.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_16x128b_x8(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x128b.x8.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15])
+        : "memory");
+}
+
+// the tcgen05.ld above complete (registers tied so that no use moves above)
+template <int N>
+__device__ __forceinline__ void tmem_ld_wait_n(uint32_t (&v)[N]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(v[i]));
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -306,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 mbar_init(v_full(i), 1);
                 mbar_init(v_empty(i), 1);
                 mbar_init(s_full(i), 1);
-                mbar_init(p_full(i), 4);  // one arrival per softmax warp
+                mbar_init(p_full(i), kSoftmaxWarps);  // one arrival per softmax warp
                 mbar_init(o_ready(i), 1);
             }
             mbar_init(drain(0), 1);
@@ -494,27 +555,36 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue
-        const int sub = warp & 3;  // TMEM sub-partition: lanes 32 sub ..
-        const int r = sub * 32 + lane;          // query row within the block
-        const uint32_t lane_base = tmem + (static_cast<uint32_t>(sub * 32) << 16);
-        const float c = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
+        // Two warps per TMEM sub-partition: warp (sub, hh) takes the 16 rows
+        // 32 sub + 16 hh .. + 15 of the block.  Thread (g, c) = (lane / 4,
+        // lane % 4) holds rows g and g + 8 of them at keys 8 j + 2 c and
+        // 8 j + 2 c + 1 (16x256b loads), so a row's max and sum combine over
+        // the four threads of a quad with two shuffles; its P pairs (key
+        // pair 4 j + c) go back with one 16x128b store.
+        const int sw = warp - kFirstSoftmaxWarp;
+        const int sub = warp & 3;
+        const int rb = sub * 32 + (sw >> 2) * 16;  // first row of the warp within the block
+        const int g = lane >> 2, c = lane & 3;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(rb) << 16);
+        const float cs = 1.4426950408889634f * p.scale;  // log2(e) / sqrt(d)
         bool ok = run;
         JobCursor cur;
-        uint32_t g = 0;
+        uint32_t gb = 0;
         for (int64_t t = t_first; ok && t < njobs; t += t_step) {
             const AttnJob jb = job_at(p, t, lane, cur);
             if (!jb.valid) break;
             int b_first, nblk;
             key_range(jb, W, b_first, nblk);
-            const int i = jb.q0 + r;  // query token
-            // Running max m (log2 units, scale folded in) and sum l.  The max is
-            // raised lazily: only when a block's max exceeds it by more than 8
-            // (p <= 2^8 otherwise), so O is rescaled rarely; O and l always use
-            // the same m, so the final O / l is exact either way.
-            float m = kMaskedScore, l = 0.0f;
-            for (int j = 0; ok && j < nblk; ++j, ++g) {
-                const uint32_t b = g & 1u;
-                if (!wait_warp(s_full(b), (g >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
+            const int i0 = jb.q0 + rb + g;  // query tokens of rows g and g + 8
+            // Running max m (log2 units, scale folded in) and this thread's
+            // part of the sum l, per row.  The max is raised lazily: only when
+            // a block's max exceeds it by more than 8 (p <= 2^8 otherwise), so
+            // O is rescaled rarely; O and l always use the same m, so the
+            // final O / l is exact either way.
+            float m0 = kMaskedScore, m1 = kMaskedScore, l0 = 0.0f, l1 = 0.0f;
+            for (int j = 0; ok && j < nblk; ++j, ++gb) {
+                const uint32_t b = gb & 1u;
+                if (!wait_warp(s_full(b), (gb >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -523,136 +593,137 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // every key of the block allowed for every query of the block
                 const bool interior = kbase + kBKV - 1 <= jb.q0 && kbase > jb.q0 + kBQ - 1 - W;
                 const uint32_t s_tm = lane_base + L::S_COL + b * kBKV;
-                // the row's scores, read once; masked keys become -inf, so
-                // their p = 2^(-inf) is exactly 0 with no compare in the exp loop
-                uint32_t v[kBKV / 32][32];
+                uint32_t v[32];
+                tmem_ld_16x256b_x8(s_tm, v);
+                tmem_ld_wait_n(v);
+                if (!interior) {
+                    // allowed key offsets for the two rows: lo .. hi (masked
+                    // keys become -inf, so their p = 2^(-inf) is exactly 0)
+                    const int hi0 = i0 - kbase, lo0 = hi0 - W + 1;
 #pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_32x32b_x32(s_tm + ch * 32, v[ch]);
+                    for (int jj = 0; jj < 8; ++jj)
 #pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) tmem_ld_wait(v[ch]);
-                // allowed key offsets in the block for query i: lo .. hi (keys past
-                // the end of the sequence only meet rows past it, never stored)
-                const int hi = i - kbase, lo = i - W + 1 - kbase;
-                // live[ch]: some lane of the warp has an allowed key in chunk ch
-                bool live[kBKV / 32];
-#pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) {
-                    live[ch] = interior || __any_sync(0xffffffffu, hi >= ch * 32 && lo <= ch * 32 + 31);
-                    if (!interior && live[ch] &&
-                        __any_sync(0xffffffffu, hi < ch * 32 + 31 || lo > ch * 32)) {
-#pragma unroll
-                        for (int t = 0; t < 32; ++t) {
-                            const int k = ch * 32 + t;
-                            if (k > hi || k < lo) v[ch][t] = 0xFF800000u;
+                        for (int e = 0; e < 2; ++e) {
+                            const int k = 8 * jj + 2 * c + e;
+                            if (k > hi0 || k < lo0) v[4 * jj + e] = 0xFF800000u;
+                            if (k > hi0 + 8 || k < lo0 + 8) v[4 * jj + 2 + e] = 0xFF800000u;
                         }
-                    }
                 }
-                float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) {
-                    if (!live[ch]) continue;
-#pragma unroll
-                    for (int t = 0; t < 32; t += 8) {
-#pragma unroll
-                        for (int u = 0; u < 4; ++u)
-                            mx[u] = fmax3(mx[u], __uint_as_float(v[ch][t + 2 * u]),
-                                          __uint_as_float(v[ch][t + 2 * u + 1]));
-                    }
+                for (int jj = 0; jj < 8; ++jj) {
+                    mx0 = fmax3(mx0, __uint_as_float(v[4 * jj]), __uint_as_float(v[4 * jj + 1]));
+                    mx1 = fmax3(mx1, __uint_as_float(v[4 * jj + 2]), __uint_as_float(v[4 * jj + 3]));
                 }
-                const float mb = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c;  // c > 0
-                const bool raise = mb > m + 8.0f;
-                const float m_new = raise ? mb : m;
-                const float alpha = ex2(m - m_new);
-                const float nm = -m_new;
-                float2 sum[2] = {make_float2(0.0f, 0.0f), make_float2(0.0f, 0.0f)};
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+                const float mb0 = mx0 * cs, mb1 = mx1 * cs;  // cs > 0
+                const bool raise0 = mb0 > m0 + 8.0f, raise1 = mb1 > m1 + 8.0f;
+                const float mn0 = raise0 ? mb0 : m0, mn1 = raise1 ? mb1 : m1;
+                const float alpha0 = ex2(m0 - mn0), alpha1 = ex2(m1 - mn1);
+                float2 sum0 = make_float2(0.0f, 0.0f), sum1 = make_float2(0.0f, 0.0f);
+                uint32_t pk[16];
 #pragma unroll
-                for (int ch = 0; ch < kBKV / 32; ++ch) {
-                    uint32_t pk[16];
-                    if (live[ch]) {
-#pragma unroll
-                        for (int t = 0; t < 16; ++t) {
-                            // p = 2^(s c - m) for a key pair: one paired FMA, two ex2
-                            float2 e = ffma2(make_float2(__uint_as_float(v[ch][2 * t]),
-                                                         __uint_as_float(v[ch][2 * t + 1])), c, nm);
-                            e.x = ex2(e.x);
-                            e.y = ex2(e.y);
-                            sum[t & 1] = fadd2(sum[t & 1], e);
-                            pk[t] = pack_bf16x2_rn(e.x, e.y);
-                        }
-                    } else {
-#pragma unroll
-                        for (int t = 0; t < 16; ++t) pk[t] = 0u;
-                    }
-                    tmem_st_32x32b_x16(s_tm + ch * 16, pk);
+                for (int jj = 0; jj < 8; ++jj) {
+                    // p = 2^(s c - m) for a key pair of each row: a paired FMA, two ex2
+                    float2 e0 = ffma2(make_float2(__uint_as_float(v[4 * jj]),
+                                                  __uint_as_float(v[4 * jj + 1])), cs, -mn0);
+                    float2 e1 = ffma2(make_float2(__uint_as_float(v[4 * jj + 2]),
+                                                  __uint_as_float(v[4 * jj + 3])), cs, -mn1);
+                    e0.x = ex2(e0.x);
+                    e0.y = ex2(e0.y);
+                    e1.x = ex2(e1.x);
+                    e1.y = ex2(e1.y);
+                    sum0 = fadd2(sum0, e0);
+                    sum1 = fadd2(sum1, e1);
+                    pk[2 * jj] = pack_bf16x2_rn(e0.x, e0.y);
+                    pk[2 * jj + 1] = pack_bf16x2_rn(e1.x, e1.y);
                 }
+                tmem_st_16x128b_x8(s_tm, pk);  // P of block gb over the first half of its S
                 // rescale O (the sum over the job's blocks before j) to the new
-                // max, once the PV product of block g - 1 has completed
-                if (j > 0 && __any_sync(0xffffffffu, raise)) {
-                    if (!wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
+                // max, once the PV product of block gb - 1 has completed
+                if (j > 0 && __any_sync(0xffffffffu, raise0 || raise1)) {
+                    if (!wait_warp(o_ready((gb - 1) & 1u), ((gb - 1) >> 1) & 1u, abort_flag,
+                                   p.status, p.wait_ns)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
 #pragma unroll 1
                     for (int ch = 0; ch < kD / 32; ++ch) {
-                        uint32_t o[32];
-                        tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
-                        tmem_ld_wait(o);
+                        uint32_t o[16];
+                        tmem_ld_16x256b_x4(lane_base + L::O_COL + ch * 32, o);
+                        tmem_ld_wait_n(o);
 #pragma unroll
-                        for (int t = 0; t < 32; ++t)
-                            o[t] = __float_as_uint(__uint_as_float(o[t]) * alpha);
-                        tmem_st_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
+                        for (int jj = 0; jj < 4; ++jj) {
+                            o[4 * jj] = __float_as_uint(__uint_as_float(o[4 * jj]) * alpha0);
+                            o[4 * jj + 1] = __float_as_uint(__uint_as_float(o[4 * jj + 1]) * alpha0);
+                            o[4 * jj + 2] = __float_as_uint(__uint_as_float(o[4 * jj + 2]) * alpha1);
+                            o[4 * jj + 3] = __float_as_uint(__uint_as_float(o[4 * jj + 3]) * alpha1);
+                        }
+                        tmem_st_16x256b_x4(lane_base + L::O_COL + ch * 32, o);
                     }
                 }
-                l = l * alpha + ((sum[0].x + sum[1].x) + (sum[0].y + sum[1].y));
-                m = m_new;
+                l0 = l0 * alpha0 + (sum0.x + sum0.y);
+                l1 = l1 * alpha1 + (sum1.x + sum1.y);
+                m0 = mn0;
+                m1 = mn1;
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(p_full(b));  // P of block g written over its S
+                if (lane == 0) mbar_arrive(p_full(b));  // P of block gb written over its S
             }
             // ---- epilogue: O / l -> bf16.  The next job's first PV product,
             // which overwrites O, waits for P of that job, which these warps
             // write only after this epilogue has read O.
-            if (!ok || !wait_warp(o_ready((g - 1) & 1u), ((g - 1) >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
+            if (!ok || !wait_warp(o_ready((gb - 1) & 1u), ((gb - 1) >> 1) & 1u, abort_flag, p.status, p.wait_ns)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const float inv = l > 0.0f ? 1.0f / l : 0.0f;
-            // Each 32-column chunk goes through the warp's staging buffer, so
-            // that a store instruction writes 8 rows x 64 contiguous bytes
-            // rather than 32 rows x 16: 16-byte unit u of row q sits at unit
-            // u ^ ((q >> 1) & 3), which keeps both sides at the minimum of
-            // four shared-memory wavefronts.
-            uint8_t* stage = smem + L::STAGE_OFF + sub * L::STAGE_WARP;
-            const int rows_left = jb.se - (jb.q0 + sub * 32);  // rows of this warp to store
+            // the rows' sums over the quad's four parts
+            l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+            l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+            const float inv0 = l0 > 0.0f ? 1.0f / l0 : 0.0f;
+            const float inv1 = l1 > 0.0f ? 1.0f / l1 : 0.0f;
+            // Each 32-column chunk of the warp's 16 rows goes through its
+            // staging buffer (16 rows x 64 bytes), so that a store instruction
+            // writes 8 rows x 64 contiguous bytes: 16-byte unit u of row q sits
+            // at unit u ^ ((q >> 1) & 3), which puts the 32 four-byte writes of
+            // a staging store on distinct banks.
+            uint8_t* stage = smem + L::STAGE_OFF + sw * L::STAGE_WARP;
+            uint32_t* stage32 = reinterpret_cast<uint32_t*>(stage);
+            const int rows_left = jb.se - (jb.q0 + rb);  // rows of this warp to store
             __nv_bfloat16* obase = reinterpret_cast<__nv_bfloat16*>(p.out) +
-                                   static_cast<int64_t>(jb.q0 + sub * 32) * Hd + jb.h * kD;
+                                   static_cast<int64_t>(jb.q0 + rb) * Hd + jb.h * kD;
+            const int sw0 = (g >> 1) & 3;  // rows g and g + 8 share the swizzle
 #pragma unroll 1
             for (int ch = 0; ch < kD / 32; ++ch) {
-                uint32_t o[32];
-                tmem_ld_32x32b_x32(lane_base + L::O_COL + ch * 32, o);
-                tmem_ld_wait(o);
+                uint32_t o[16];
+                tmem_ld_16x256b_x4(lane_base + L::O_COL + ch * 32, o);
+                tmem_ld_wait_n(o);
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const uint32_t* w8 = &o[8 * u];
-                    uint4 w;
-                    w.x = pack_bf16x2_rn(__uint_as_float(w8[0]) * inv, __uint_as_float(w8[1]) * inv);
-                    w.y = pack_bf16x2_rn(__uint_as_float(w8[2]) * inv, __uint_as_float(w8[3]) * inv);
-                    w.z = pack_bf16x2_rn(__uint_as_float(w8[4]) * inv, __uint_as_float(w8[5]) * inv);
-                    w.w = pack_bf16x2_rn(__uint_as_float(w8[6]) * inv, __uint_as_float(w8[7]) * inv);
-                    *reinterpret_cast<uint4*>(stage + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) = w;
+                for (int jj = 0; jj < 4; ++jj) {
+                    // columns 8 jj + 2 c, + 1: word 4 jj + c of the row, in unit jj
+                    const int word = 4 * (jj ^ sw0) + c;
+                    stage32[g * 16 + word] = pack_bf16x2_rn(__uint_as_float(o[4 * jj]) * inv0,
+                                                            __uint_as_float(o[4 * jj + 1]) * inv0);
+                    stage32[(g + 8) * 16 + word] =
+                        pack_bf16x2_rn(__uint_as_float(o[4 * jj + 2]) * inv1,
+                                       __uint_as_float(o[4 * jj + 3]) * inv1);
                 }
                 __syncwarp();
 #pragma unroll
-                for (int it = 0; it < 4; ++it) {
+                for (int it = 0; it < 2; ++it) {
                     const int q = it * 8 + (lane >> 2), u = lane & 3;
                     const uint4 w = *reinterpret_cast<const uint4*>(stage + q * 64 +
                                                                     ((u ^ ((q >> 1) & 3)) << 4));
                     if (q < rows_left &&
-                        dbg_check(jb.q0 + sub * 32 + q < jb.se && jb.q0 + sub * 32 + q >= jb.ss,
-                                  p.status))
+                        dbg_check(jb.q0 + rb + q < jb.se && jb.q0 + rb + q >= jb.ss, p.status))
                         *reinterpret_cast<uint4*>(obase + static_cast<int64_t>(q) * Hd + ch * 32 + u * 8) = w;
                 }
                 __syncwarp();
