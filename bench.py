@@ -57,7 +57,7 @@ NCU_TRAFFIC = {
     ("gemv32", "gemvtc", "b81ddd27f1e19156"): 0.32655e9 + 0.00362e9,
     # attention prefill per 8 pairs of 1024 tokens x 96 heads (full capture of
     # one 8-pair launch); scaled by pairs / 8 for the benched launch
-    ("attention", "attn", "3294a8d7153edae5"): 0.8125e9 + 0.1834e9,
+    ("attention", "attn", "f94e5ad5312cd435"): 0.8716e9 + 0.1923e9,
 }
 
 KERNEL_FILES = {"ts": ("ts_gemm.cu", "dequant.cuh", "ptx.cuh"),
