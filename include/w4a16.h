@@ -3,8 +3,8 @@
  * layer library.
  *
  * The operation.  The paper scores protein-ligand pairs with a 175B-class
- * decoder run "4-bit pre-quantized" with "mixed-precision quantization"
- * (Sec. 3.1, Sec. 4.1), in batches through its prediction module
+ * decoder whose weights are quantised to 4 bits ahead of time, with mixed
+ * precision (Sec. 3.1, Sec. 4.1), run in batches through its prediction module
  * (Sec. 3.3).  On the prefill path the linear layers (fused QKV, attention
  * output, MLP up, MLP down) are y = x W^T with W held at 4 bits.  The paper
  * gives no format; this library fixes one:
@@ -174,7 +174,7 @@ int w4a16_stack_graph_destroy(w4a16_stack_graph* graph);
 
 /*
  * wd = dequant(w_packed, scales) as bf16 [N, K] (device): the 4-bit weights
- * of the pre-quantised model (Sec. 4.1; "mixed-precision quantization",
+ * of the pre-quantised model (Sec. 4.1; mixed-precision quantisation,
  * Sec. 3.1) brought back to the precision the matmul runs in, with the
  * format and rounding stated at the top of this file.  The same unpack and
  * rounding as inside the tcgen05 GEMM, exported so that it can be compared
